@@ -1,0 +1,176 @@
+"""Seeded synthetic MAR-shaped workloads.
+
+The paper evaluates on ImageNet 256x256 class-conditional generation with
+trained MAR-B/L/H weights (Sec. 4.1). Neither the dataset nor the weights are
+available, so every input here is synthetic with the paper's shapes: 64 buffer
+(class) tokens prepended to 256 KL-16 image tokens of latent dimension 16, 1000
+classes, 64-step decoding. Weights are N(0, 0.02); LayerNorm gains are
+1 + N(0, 0.1) and shifts N(0, 0.02) so that a swapped gain/shift is visible.
+
+Generators (numpy PCG64, fixed seeds):
+  weights            seed 0 (+ config-independent stream order, see make_weights)
+  class labels       seed 1, uniform over [0, n_classes)
+  decode order       seed 2, one permutation of the image positions per
+                     cond/uncond pair
+  token latents      seed 3, one N(0, 1) latent per (pair, image position),
+                     revealed once that position is decoded
+
+bf16 configurations store weights as bf16: `round_bf16` maps fp32 values to
+the nearest bf16 value (ties to even) and keeps them in fp32 containers, so
+both sides read identical numbers.
+"""
+import math
+
+import numpy as np
+
+# Model/workload shapes. `batch` counts cond/uncond pairs (B); the forward runs
+# rows = 2B (both pathways) or B (condition-cache reuse step).
+CONFIGS = {
+    # 2 blocks, width 256, 4 heads, 16 buffer + 64 image tokens, one pair, fp32.
+    "tiny": dict(depth=2, width=256, heads=4, mlp_ratio=4, n_buffer=16, n_img=64,
+                 token_dim=16, n_classes=1000, batch=1, sel_layers=1, dtype="fp32",
+                 steps=64, k0=4, tau=9, tau_cfg=9, ratio=0.25),
+    # 12 encoder + 12 decoder blocks, width 768, 12 heads, B = 32.
+    "mar_b": dict(depth=24, width=768, heads=12, mlp_ratio=4, n_buffer=64, n_img=256,
+                  token_dim=16, n_classes=1000, batch=32, sel_layers=3, dtype="bf16",
+                  steps=64, k0=4, tau=9, tau_cfg=2, ratio=50 / 320),
+    # 16 + 16 blocks, width 1024, 16 heads, B = 64.
+    "mar_l": dict(depth=32, width=1024, heads=16, mlp_ratio=4, n_buffer=64, n_img=256,
+                  token_dim=16, n_classes=1000, batch=64, sel_layers=3, dtype="bf16",
+                  steps=64, k0=4, tau=9, tau_cfg=9, ratio=50 / 320),
+    # 20 + 20 blocks, width 1280, 16 heads (head dim 80), B = 128.
+    "mar_h": dict(depth=40, width=1280, heads=16, mlp_ratio=4, n_buffer=64, n_img=256,
+                  token_dim=16, n_classes=1000, batch=128, sel_layers=3, dtype="bf16",
+                  steps=64, k0=4, tau=9, tau_cfg=9, ratio=50 / 320),
+    # MAR-L shapes at 32x32 latents: 64 + 1024 tokens, B = 16, 25 % recompute.
+    "hires": dict(depth=32, width=1024, heads=16, mlp_ratio=4, n_buffer=64, n_img=1024,
+                  token_dim=16, n_classes=1000, batch=16, sel_layers=3, dtype="bf16",
+                  steps=64, k0=4, tau=9, tau_cfg=0, ratio=0.25),
+}
+
+
+def config(name, **overrides):
+    """Return a copy of a named configuration with derived fields filled in."""
+    c = dict(CONFIGS[name])
+    c.update(overrides)
+    c["name"] = name
+    c["T"] = c["n_buffer"] + c["n_img"]
+    c["head_dim"] = c["width"] // c["heads"]
+    c["ln_eps"] = 1e-6
+    c.setdefault("criterion", "value")
+    return c
+
+
+def n_compute(cfg, ratio=None):
+    """Tokens recomputed per row: round-half-up(ratio * T)."""
+    r = cfg["ratio"] if ratio is None else ratio
+    return int(math.floor(r * cfg["T"] + 0.5))
+
+
+def round_bf16(x):
+    """Nearest bf16 value (ties to even) of each fp32 element, as fp32."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
+    u = (u + (((u >> 16) & 1) + 0x7FFF)) & 0xFFFF0000
+    return u.astype(np.uint32).view(np.float32)
+
+
+def _normal(rng, shape, std):
+    return (rng.standard_normal(shape, dtype=np.float32) * np.float32(std)).astype(np.float32)
+
+
+def make_weights(cfg, seed=0):
+    """Random-init weights of the MAR-shaped transformer (nn.Linear layout [out, in]).
+
+    Returns a dict of fp32 arrays; for bf16 configurations every value is
+    already bf16-representable.
+    """
+    rng = np.random.Generator(np.random.PCG64(seed))
+    D, T, H4 = cfg["width"], cfg["T"], cfg["width"] * cfg["mlp_ratio"]
+    w = {
+        "pos_emb": _normal(rng, (T, D), 0.02),
+        "class_emb": _normal(rng, (cfg["n_classes"], D), 0.02),
+        "mask_emb": _normal(rng, (D,), 0.02),
+        "embed_w": _normal(rng, (D, cfg["token_dim"]), 0.02),
+        "embed_b": _normal(rng, (D,), 0.02),
+        "lnf_g": (1.0 + _normal(rng, (D,), 0.1)).astype(np.float32),
+        "lnf_b": _normal(rng, (D,), 0.02),
+        "blocks": [],
+    }
+    for _ in range(cfg["depth"]):
+        w["blocks"].append({
+            "ln1_g": (1.0 + _normal(rng, (D,), 0.1)).astype(np.float32),
+            "ln1_b": _normal(rng, (D,), 0.02),
+            "w_qkv": _normal(rng, (3 * D, D), 0.02),
+            "b_qkv": _normal(rng, (3 * D,), 0.02),
+            "w_o": _normal(rng, (D, D), 0.02),
+            "b_o": _normal(rng, (D,), 0.02),
+            "ln2_g": (1.0 + _normal(rng, (D,), 0.1)).astype(np.float32),
+            "ln2_b": _normal(rng, (D,), 0.02),
+            "w1": _normal(rng, (H4, D), 0.02),
+            "b1": _normal(rng, (H4,), 0.02),
+            "w2": _normal(rng, (D, H4), 0.02),
+            "b2": _normal(rng, (D,), 0.02),
+        })
+    if cfg["dtype"] == "bf16":
+        for k in list(w):
+            if k != "blocks":
+                w[k] = round_bf16(w[k])
+        for b in w["blocks"]:
+            for k in b:
+                b[k] = round_bf16(b[k])
+    return w
+
+
+def make_labels(cfg, seed=1):
+    rng = np.random.Generator(np.random.PCG64(seed))
+    return rng.integers(0, cfg["n_classes"], size=cfg["batch"], dtype=np.int64).astype(np.int32)
+
+
+def make_order(cfg, seed=2):
+    """Decode order: one permutation of image positions per pair, [B, n_img]."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    return np.stack([rng.permutation(cfg["n_img"]) for _ in range(cfg["batch"])]).astype(np.int32)
+
+
+def make_latent_table(cfg, seed=3):
+    """Latent revealed for each (pair, image position) once decoded, [B, n_img, token_dim]."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    return rng.standard_normal((cfg["batch"], cfg["n_img"], cfg["token_dim"]), dtype=np.float32)
+
+
+def mask_counts(steps, n_img):
+    """Masked image tokens left after each decoding step (cosine schedule, as in MAR/MaskGIT).
+
+    m[k] = floor(n_img * cos(pi/2 * (k+1)/steps)), clamped so that every step
+    decodes at least one token and the last step decodes the rest (m[-1] = 0).
+    This is workload structure for the synthetic driver, not part of LazyMAR.
+    """
+    m, prev = [], n_img
+    for k in range(steps):
+        if k == steps - 1:
+            cur = 0
+        else:
+            cur = int(math.floor(n_img * math.cos(math.pi / 2 * (k + 1) / steps)))
+            cur = max(1, min(cur, prev - 1))
+        m.append(cur)
+        prev = cur
+    return m
+
+
+def step_state(cfg, order, table, n_decoded):
+    """Inputs of one forward: latents [B, n_img, token_dim] fp32, mask [B, n_img] u8 (1 = masked).
+
+    The first `n_decoded` positions of each pair's order are decoded and carry
+    their latent; the rest are masked (their latent entries are zero).
+    """
+    B, n = order.shape
+    mask = np.ones((B, n), dtype=np.uint8)
+    for b in range(B):
+        mask[b, order[b, :n_decoded]] = 0
+    lat = np.where(mask[:, :, None] == 0, table, 0.0).astype(np.float32)
+    return lat, mask
+
+
+def tiny_state(cfg, order, table, before=24, after=32):
+    """The tiny workload: a forward with 24 decoded tokens, then one with 8 more."""
+    return step_state(cfg, order, table, before), step_state(cfg, order, table, after)
