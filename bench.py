@@ -1,0 +1,397 @@
+"""Benchmark: MAR-B-shaped 64-step decode with LazyMAR's caches on one GB300.
+
+One benchmark step is one whole decode of a batch: 64 decoding steps of a
+MAR-B-shaped transformer (24 blocks, width 768, 12 heads, 64 buffer + 256
+image tokens) over 32 class-conditional + 32 unconditional rows, following the
+periodic cache-reuse-refreshment schedule (full steps for k < 4 and every 9
+steps after, cached steps recomputing 50 of 320 tokens per row in between, the
+condition cache reused on every other cached step). Inputs (latents and masks
+of all 64 steps, labels) are synthetic and seeded, resident in HBM before the
+timed region; weights are random-init bf16 of the MAR-B shapes.
+
+Prints one JSON line (rank 0): images/s of the whole job, decoding steps/s, the
+full-recompute decode on the same GPU, per-kernel-class device time from CUDA
+events recorded around each launch on its stream, the GEMM roofline against
+the measured bf16 peak, an end-to-end figure through the C ABI with host
+buffers, SM clocks sampled during the timed region, and the CPU oracle timed on
+a bounded sample of the same workload.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Multi-GPU (torchrun, one process per GPU): cond/uncond pairs are independent,
+so every rank decodes its own batch (weak scaling, no data-path collective);
+the timed region is bracketed by barriers and the maximum over ranks is used.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "MAR-B-shaped 256-token decode: steps/sec and images/sec at 1 GB300; tensor-pipe % of peak"
+GAMMA = 3.0
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def workload(cfg):
+    n = synth.n_compute(cfg)
+    return {
+        "workload": "MAR-B-shaped 64-step LazyMAR decode (24 blocks, width 768, 12 heads, 64+256 tokens)",
+        "batch_pairs": cfg["batch"], "rows": 2 * cfg["batch"], "tokens": cfg["T"],
+        "recompute": "%d/%d tokens per row" % (n, cfg["T"]),
+        "schedule": "full for k<%d and every %d steps; cond cache reused every other cached step" % (
+            cfg["k0"], cfg["tau"]),
+        "decoding_steps": cfg["steps"],
+        "l2": "no flush: the per-step working set (0.34 GB weights + 1.3 GB K/V cache) exceeds the 129 MB L2",
+    }
+
+
+def schedule(cfg, plan_fn):
+    return [plan_fn(k, cfg["k0"], cfg["tau"], cfg["tau_cfg"], True) for k in range(cfg["steps"])]
+
+
+def decode_inputs(cfg, seed_offset):
+    """Latents and masks of every decoding step for one batch (numpy)."""
+    order = synth.make_order(cfg, seed=2 + seed_offset)
+    table = synth.make_latent_table(cfg, seed=3 + seed_offset)
+    labels = synth.make_labels(cfg, seed=1 + seed_offset)
+    m = synth.mask_counts(cfg["steps"], cfg["n_img"])
+    lats, masks = [], []
+    for k in range(cfg["steps"]):
+        n_dec = cfg["n_img"] - (m[k - 1] if k > 0 else cfg["n_img"])
+        lat, mask = synth.step_state(cfg, order, table, n_dec)
+        lats.append(lat)
+        masks.append(mask)
+    return np.stack(lats), np.stack(masks), labels
+
+
+# --------------------------------------------------------------------------
+# Clocks sampled during the timed region
+# --------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ["clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.hw_slowdown",
+              "clocks_event_reasons.hw_thermal_slowdown", "clocks_event_reasons.sw_thermal_slowdown",
+              "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + ",".join(self.FIELDS),
+                 "--format=csv,noheader,nounits", "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.t.join(timeout=5)
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[3:7]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------
+# CPU oracle baseline (bounded sample)
+# --------------------------------------------------------------------------
+
+def oracle_sample(cfg, plan):
+    """Times the oracle on one cond/uncond pair: a full step, a cached step with
+    both pathways and a condition-cache reuse step; scales to images/s with the
+    schedule's step counts."""
+    import oracle as O
+    c1 = dict(cfg, batch=1)
+    W = synth.make_weights(c1)
+    lat, mask, labels = decode_inputs(c1, 0)
+    N = synth.n_compute(cfg)
+    cache = O.Cache(c1, 1)
+    t0 = time.perf_counter()
+    O.full_step(c1, W, cache, lat[10], mask[10], labels, GAMMA)
+    t1 = time.perf_counter()
+    O.cached_step(c1, W, cache, lat[11], mask[11], labels, N, False, GAMMA)
+    t2 = time.perf_counter()
+    O.cached_step(c1, W, cache, lat[12], mask[12], labels, N, True, GAMMA)
+    t3 = time.perf_counter()
+    n_full = sum(1 for f, r in plan if f)
+    n_reuse = sum(1 for f, r in plan if not f and r)
+    n_both = len(plan) - n_full - n_reuse
+    sec_per_image = n_full * (t1 - t0) + n_both * (t2 - t1) + n_reuse * (t3 - t2)
+    cores = int(os.environ.get("OPENBLAS_NUM_THREADS") or os.environ.get("OMP_NUM_THREADS") or os.cpu_count())
+    return {
+        "value": 1.0 / sec_per_image, "unit": "images/s", "cores": cores, "kind": "oracle",
+        "sample": "one cond/uncond pair: 1 full + 1 cached + 1 cond-reuse step (%.1f s of fp64 numpy), scaled by "
+                  "the 64-step schedule (%d full, %d cached, %d cond-reuse)" % (t3 - t0, n_full, n_both, n_reuse),
+        "sample_s": t3 - t0,
+    }
+
+
+def run_reference(args, cfg, plan):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    for _ in range(args.warmup):
+        oracle_sample(cfg, plan)
+    vals, secs = [], []
+    cb = None
+    for _ in range(args.steps):
+        cb = oracle_sample(cfg, plan)
+        vals.append(cb["value"])
+        secs.append(cb["sample_s"])
+    value = statistics.median(vals)
+    cb = dict(cb, value=value)
+    cb.pop("sample_s", None)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "images/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 / value, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": workload(cfg),
+            "cpu_baseline": cb, "e2e": {"value": value, "unit": "images/s", "h2d_bytes_per_step": 0,
+                                        "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------------
+# GPU arm
+# --------------------------------------------------------------------------
+
+def run_ours(args, cfg):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2503_12450_gb300 import build as libbuild
+    from paper_2503_12450_gb300 import lazymar as lm
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    if rank == 0:
+        libbuild.build()
+    if world > 1:
+        dist.barrier()
+    lm.lib()
+    plan = schedule(cfg, lm.lazymar_plan_step)
+
+    B, N, steps = cfg["batch"], synth.n_compute(cfg), cfg["steps"]
+    W = synth.make_weights(cfg)
+    h = lm.lazymar_create(dict(cfg, max_batch=B), W)
+    lat_np, mask_np, labels_np = decode_inputs(cfg, rank * 101)
+    lat = torch.from_numpy(lat_np).cuda()
+    mask = torch.from_numpy(mask_np).cuda()
+    labels = torch.from_numpy(labels_np).cuda()
+    guided = torch.empty((B, cfg["n_img"], cfg["width"]), dtype=torch.bfloat16, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def decode(full_only=False, host=None, step_events=None):
+        for k in range(steps):
+            full, reuse = plan[k]
+            if host is not None:
+                l_k, m_k, lab, g = host["lat"][k], host["mask"][k], host["labels"], host["guided"]
+            else:
+                l_k, m_k, lab, g = lat[k], mask[k], labels, guided
+            if step_events is not None:
+                step_events[k][0].record(stream)
+            if full or full_only:
+                lm.lazymar_full_step(h, l_k, m_k, lab, B, GAMMA, None, g, stream)
+            else:
+                lm.lazymar_cached_step(h, l_k, m_k, lab, B, N, reuse, GAMMA, None, None, None, g, stream)
+            if step_events is not None:
+                step_events[k][1].record(stream)
+        if host is not None:
+            stream.synchronize()  # the caller reads the last step's guided output
+
+    def timed(fn, k_steps):
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0 = time.perf_counter()
+        e0.record(stream)
+        for _ in range(k_steps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+        ms = e0.elapsed_time(e1)
+        if world > 1:
+            t = torch.tensor([ms, wall * 1000.0], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ms, wall = float(t[0]), float(t[1]) / 1000.0
+            dist.barrier()
+        return ms, wall
+
+    for _ in range(args.warmup):
+        decode()
+    lm.lazymar_sync(h, stream)
+
+    # 1) the headline: device-resident inputs, CUDA events around K decodes
+    lm.lazymar_reset_stats(h)
+    with ClockSampler(local) as clocks:
+        ms, wall = timed(decode, args.steps)
+    st = lm.lazymar_get_stats(h)
+    launches = sum(v["launches"] for v in st.values())
+    lm.lazymar_sync(h, stream)
+    ms_per_step = ms / args.steps
+    images_per_s = world * B * args.steps / (ms / 1000.0)
+
+    # 2) per-kernel device time: events around every launch (separate pass)
+    lm.lazymar_reset_stats(h)
+    lm.lazymar_set_profiling(h, True)
+    step_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    kind_ms = {"full": [], "cached": [], "cached_reuse": []}
+    for _ in range(max(1, min(args.steps, 3))):
+        decode(step_events=step_ev)
+        torch.cuda.synchronize()
+        for k in range(steps):
+            full, reuse = plan[k]
+            kind = "full" if full else ("cached_reuse" if reuse else "cached")
+            kind_ms[kind].append(step_ev[k][0].elapsed_time(step_ev[k][1]))
+    prof = lm.lazymar_get_stats(h)
+    lm.lazymar_set_profiling(h, False)
+    lm.lazymar_sync(h, stream)
+
+    # 3) full recompute on the same GPU (every decoding step a full step)
+    for _ in range(1):
+        decode(full_only=True)
+    ms_full, _ = timed(lambda: decode(full_only=True), args.steps)
+    full_images_per_s = world * B * args.steps / (ms_full / 1000.0)
+
+    # 4) end to end through the C ABI with host buffers (pinned), copies inside
+    host = {"lat": lat.cpu().pin_memory(), "mask": mask.cpu().pin_memory(), "labels": labels.cpu().pin_memory(),
+            "guided": torch.empty(tuple(guided.shape), dtype=torch.bfloat16).pin_memory()}
+    decode(host=host)
+    ms_e2e, _ = timed(lambda: decode(host=host), args.steps)
+    e2e_images_per_s = world * B * args.steps / (ms_e2e / 1000.0)
+    h2d = steps * (lat[0].numel() * 4 + mask[0].numel() + labels.numel() * 4)
+    d2h = steps * guided.numel() * 2
+    lm.lazymar_sync(h, stream)
+
+    if rank != 0:
+        h.close()
+        dist.destroy_process_group()
+        return
+
+    pk, src = peaks()
+    peak_tf = pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
+    g = prof["gemm"]
+    gemm_tflops = g["flops"] / (g["ms"] / 1000.0) / 1e12 if g["ms"] > 0 else None
+    total_ms = sum(v["ms"] for v in prof.values())
+    kernels = {}
+    for name, v in prof.items():
+        if v["timed_launches"] == 0:
+            continue
+        kernels[name] = {"launches": v["timed_launches"], "ms": round(v["ms"], 3),
+                         "share": round(v["ms"] / total_ms, 4) if total_ms else None,
+                         "tflops": round(v["flops"] / (v["ms"] / 1e3) / 1e12, 2) if v["flops"] and v["ms"] else None,
+                         "gbs": round(v["bytes"] / (v["ms"] / 1e3) / 1e9, 1) if v["ms"] else None}
+    traffic = None
+    tpath = os.path.join(ROOT, "profiles", "gemm_traffic.json")
+    if os.path.exists(tpath):
+        with open(tpath) as f:
+            traffic = json.load(f).get("bytes_per_launch")
+    line = {
+        "metric": METRIC, "value": images_per_s, "unit": "images/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded latents/masks, random-init MAR-B weights)",
+        "config": workload(cfg),
+        "decoding_steps_per_s": world * steps * args.steps / (ms / 1000.0),
+        "step_ms": {k: round(statistics.mean(v), 3) for k, v in kind_ms.items() if v},
+        "full_recompute": {"value": full_images_per_s, "unit": "images/s", "ms_per_step": ms_full / args.steps,
+                           "speedup": images_per_s / full_images_per_s},
+        "roofline": {"bound": "tensor", "kernel": "gemm_bf16_tc (tcgen05)", "achieved": gemm_tflops,
+                     "peak": peak_tf, "unit": "TFLOP/s",
+                     "frac": (gemm_tflops / peak_tf) if gemm_tflops else None,
+                     "peak_source": "%s bf16 sustained" % src, "traffic": traffic},
+        "kernels": kernels,
+        "e2e": {"value": e2e_images_per_s, "unit": "images/s", "h2d_bytes_per_step": int(h2d),
+                "d2h_bytes_per_step": int(d2h)},
+        "gpu_launches": int(launches),
+        "clocks": clocks.summary(),
+        "wall_s": wall,
+    }
+    if not args.no_cpu_baseline and world == 1:
+        line["cpu_baseline"] = oracle_sample(cfg, plan)
+        line["cpu_baseline"].pop("sample_s", None)
+    print(json.dumps(line), flush=True)
+    h.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="mar_b")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    cfg = synth.config(args.config)
+    if args.impl == "reference":
+        import oracle as O
+        plan = [O.plan(k, cfg["k0"], cfg["tau"], cfg["tau_cfg"]) for k in range(cfg["steps"])]
+        run_reference(args, cfg, plan)
+    else:
+        run_ours(args, cfg)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,260 @@
+/*
+ * lazymar.h - C ABI of a GB300 (sm_103a) implementation of LazyMAR's cached
+ * MAR decoding step (Yan et al., "LazyMAR: Accelerating Masked Autoregressive
+ * Models via Feature Caching", ICCV 2025).
+ *
+ * A masked autoregressive (MAR) transformer is run once per decoding step over
+ * a sequence of T = n_buffer + n_img tokens per image: n_buffer conditional
+ * (class) tokens followed by the image tokens (Eq. 6; 64 + 256 tokens in the
+ * paper's setting, Sec. 4.1). Bidirectional attention (Eq. 3) rules out a KV
+ * cache, so LazyMAR caches features instead:
+ *   - token cache (Sec. 3.2.1): after the first `sel_layers` blocks, each
+ *     token's value matrix is compared with its value at the previous step
+ *     (cosine similarity, Eq. 8); only the N least similar tokens are run
+ *     through the remaining blocks (Eq. 9), attending over cached keys/values
+ *     of the other tokens, and the results are written back into the cache;
+ *   - condition cache (Sec. 3.2.2, Eq. 10): the difference between the
+ *     conditional and unconditional outputs is stored on steps that run both
+ *     classifier-free-guidance pathways and reused on steps that run only the
+ *     conditional one;
+ *   - periodic refresh (Sec. 1, Fig. 3): full steps recompute everything and
+ *     refill both caches.
+ *
+ * Conventions for every entry point
+ *   - Row layout: a batch of B cond/uncond pairs runs as rows 0..B-1
+ *     (conditional pathway of pairs 0..B-1) and B..2B-1 (unconditional pathway
+ *     of the same pairs). Feature tensors are row-major [rows, tokens, width].
+ *   - dtype: LAZYMAR_BF16 tensors hold raw bfloat16 (uint16 storage),
+ *     LAZYMAR_F32 tensors IEEE float32. Arithmetic accumulates in fp32 (fp64
+ *     for the similarity of Eq. 8).
+ *   - Pointers: unless stated otherwise a tensor pointer may be device memory or
+ *     host memory (pinned or pageable). Host buffers are staged through
+ *     library-owned device buffers with cudaMemcpyAsync on `stream`.
+ *   - stream: a cudaStream_t (NULL = legacy default stream). Calls enqueue work
+ *     and return without waiting; buffers must stay valid until the stream work
+ *     has completed. Argument errors are returned immediately and enqueue
+ *     nothing. Errors detected on the device (bounded waits that expired,
+ *     out-of-range indices or labels) are latched in a device error word and
+ *     reported by lazymar_sync / lazymar_device_check.
+ *   - No call allocates device memory except lazymar_create and
+ *     lazymar_select_tokens (stream-ordered scratch for the similarities).
+ *   - A handle is not thread-safe; distinct handles are independent.
+ */
+#ifndef LAZYMAR_H
+#define LAZYMAR_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum lazymar_status {
+  LAZYMAR_OK = 0,
+  LAZYMAR_ERR_INVALID_ARG = 1,  /* bad pointer, size or enum value */
+  LAZYMAR_ERR_OOM = 2,          /* device allocation failed */
+  LAZYMAR_ERR_CUDA = 3,         /* a CUDA runtime call or launch failed */
+  LAZYMAR_ERR_STATE = 4,        /* cached step before any full step, or batch changed */
+  LAZYMAR_ERR_TIMEOUT = 5,      /* a bounded device-side wait expired */
+  LAZYMAR_ERR_UNSUPPORTED = 6,  /* shape outside what the kernels support */
+  LAZYMAR_ERR_DEVICE = 7        /* a kernel found a bad index or label on the device */
+} lazymar_status;
+
+typedef enum lazymar_dtype { LAZYMAR_F32 = 0, LAZYMAR_BF16 = 1 } lazymar_dtype;
+
+/* Which representation of block sel_layers-1 the similarity of Eq. 8 compares:
+ * the attention value matrix (Sec. 4.4 "value matrix instead of features";
+ * default) or the block's output features (Eq. 8 as printed). */
+typedef enum lazymar_criterion {
+  LAZYMAR_CRITERION_VALUE = 0,
+  LAZYMAR_CRITERION_FEATURE = 1
+} lazymar_criterion;
+
+/* Model and capacity. width % 128 == 0, head width (width/heads) 64 or 80 for
+ * bf16 (any divisor of width up to 128 for f32), token_dim <= 64,
+ * 1 <= sel_layers <= depth, 1 <= max_batch (pairs). */
+typedef struct lazymar_config {
+  int depth;       /* transformer blocks L (encoder + decoder stacked) */
+  int width;       /* D */
+  int heads;       /* H */
+  int mlp_ratio;   /* MLP hidden = mlp_ratio * D */
+  int n_buffer;    /* conditional (class) tokens C of Eq. 6 */
+  int n_img;       /* image tokens */
+  int token_dim;   /* latent width of an image token (16 for KL-16) */
+  int n_classes;   /* rows of the class-embedding table */
+  int max_batch;   /* largest B (pairs) any step will use */
+  int sel_layers;  /* s: blocks always run in full; Eq. 8 compares block s-1 */
+  int dtype;       /* lazymar_dtype of weights, activations and caches */
+  int criterion;   /* lazymar_criterion */
+  float ln_eps;    /* LayerNorm epsilon */
+} lazymar_config;
+
+/* Weights of one pre-LN block, fp32, [out, in] layout (y = x W^T + b).
+ * Read once by lazymar_create (host or device pointers) and converted to the
+ * configured dtype (bf16: round to nearest even). */
+typedef struct lazymar_block_weights {
+  const float *ln1_g, *ln1_b;  /* [D] */
+  const float *w_qkv, *b_qkv;  /* [3D, D], [3D]; rows 0..D-1 Q, D..2D-1 K, 2D..3D-1 V */
+  const float *w_o, *b_o;      /* [D, D], [D] */
+  const float *ln2_g, *ln2_b;  /* [D] */
+  const float *w1, *b1;        /* [mlp_ratio*D, D], [mlp_ratio*D] */
+  const float *w2, *b2;        /* [D, mlp_ratio*D], [D] */
+} lazymar_block_weights;
+
+typedef struct lazymar_weights {
+  const float *pos_emb;    /* [T, D] position embedding, added at every position */
+  const float *class_emb;  /* [n_classes, D]; buffer tokens of the cond pathway */
+  const float *mask_emb;   /* [D]; masked image tokens */
+  const float *embed_w;    /* [D, token_dim]; decoded image tokens */
+  const float *embed_b;    /* [D] */
+  const float *lnf_g, *lnf_b;            /* [D] final LayerNorm */
+  const lazymar_block_weights *blocks;   /* host array of `depth` entries */
+} lazymar_weights;
+
+/* Inputs of one decoding step for B pairs (both pathways share them). */
+typedef struct lazymar_step_in {
+  const float *latents;   /* [B, n_img, token_dim] fp32; ignored where masked */
+  const uint8_t *mask;    /* [B, n_img], 1 = still masked, 0 = decoded */
+  const int32_t *labels;  /* [B] class labels in [0, n_classes) */
+  int batch;              /* B, 1 <= B <= max_batch */
+} lazymar_step_in;
+
+typedef struct lazymar_handle lazymar_handle;
+
+/* Creates a model instance on the current CUDA device: copies and converts the
+ * weights and allocates the token cache (keys/values of blocks s..L-1), the
+ * selection reference, the output cache, the condition cache and all scratch
+ * for max_batch pairs. The handle owns all of it until lazymar_destroy.
+ * Returns INVALID_ARG / UNSUPPORTED for bad configurations, OOM if the device
+ * allocation fails. */
+lazymar_status lazymar_create(const lazymar_config *cfg, const lazymar_weights *w,
+                              lazymar_handle **out);
+void lazymar_destroy(lazymar_handle *h);
+
+/* Full (refresh) step, Fig. 3 and Sec. 1 "periodic cache-reuse-refreshment":
+ * every block over every token of both pathways (2B rows); refills the token
+ * cache (C_token^l := F^l(X), Sec. 3.2.1), the selection reference and the
+ * condition cache (Eq. 10).
+ *   z_out      [2B, n_img, D] final features of the image tokens (may be NULL)
+ *   guided_out [B, n_img, D]  u + gamma (c - u) (may be NULL) */
+lazymar_status lazymar_full_step(lazymar_handle *h, const lazymar_step_in *in, float gamma,
+                                 void *z_out, void *guided_out, void *stream);
+
+/* Cached step (Sec. 3.2, Eq. 8-10). Blocks 0..s-1 run over all tokens; at
+ * block s-1 Eq. 8 picks, per row, the n_compute tokens whose value matrix is
+ * least similar to the previous step's (ties to the lower token index) and the
+ * selection reference is overwritten; blocks s..L-1 run only those tokens
+ * (their queries attend over all T keys, cached for the others, Eq. 9) and
+ * write their keys, values and output features back into the cache.
+ *   n_compute       N, 0 <= N <= T tokens recomputed per row
+ *   use_cond_cache  1: run only the conditional rows (B) and rebuild the
+ *                   unconditional output as c - delta (Sec. 3.2.2);
+ *                   0: run both pathways (2B rows) and refresh delta
+ *   idx_in          optional [rows, N] int32 caller-chosen I_compute (strictly
+ *                   increasing per row, values in [0, T)); replaces Eq. 8's
+ *                   choice (the selection reference is still updated)
+ *   idx_out         optional [rows, N] int32: the I_compute used, ascending
+ *   z_out, guided_out as for lazymar_full_step.
+ * Returns STATE before the first full step or when B differs from it. */
+lazymar_status lazymar_cached_step(lazymar_handle *h, const lazymar_step_in *in, int n_compute,
+                                   int use_cond_cache, float gamma, const int32_t *idx_in,
+                                   int32_t *idx_out, void *z_out, void *guided_out, void *stream);
+
+/* Token selection of Eq. 8 on caller buffers (device pointers only).
+ * v_cur, v_cache: [rows, T, D] in `dtype`. For every row: S_t = cosine of
+ * v_cur[t] and v_cache[t] over D (fp64 accumulation of exact products,
+ * S = dot / sqrt(max(|a|^2 |b|^2, 1e-16)), NaN counted as -inf); I_compute =
+ * the n_compute smallest S, ties to the lower index, written ascending to
+ * idx_out [rows, n_compute]. Then v_cache := v_cur. D % 8 == 0.
+ * Allocates rows*T doubles of stream-ordered scratch (cudaMallocAsync). */
+lazymar_status lazymar_select_tokens(int dtype, const void *v_cur, void *v_cache, int rows, int T,
+                                     int D, int n_compute, int32_t *idx_out, void *stream);
+
+/* Classifier-free guidance with the condition cache (Eq. 7 read as
+ * u + gamma (c - u), Eq. 10), elementwise over n elements (device pointers):
+ *   mode 0 GUIDE:   guided = u + gamma (c - u)
+ *   mode 1 REFRESH: delta := c - u; guided = u + gamma (c - u)
+ *   mode 2 REUSE:   u' = c - delta; guided = u' + gamma (c - u');
+ *                   z_uncond_out := u' (if not NULL). z_uncond is unused.
+ * guided_out may be NULL. Arithmetic in fp32. */
+enum { LAZYMAR_CFG_GUIDE = 0, LAZYMAR_CFG_REFRESH = 1, LAZYMAR_CFG_REUSE = 2 };
+lazymar_status lazymar_cfg_combine(int dtype, int mode, const void *z_cond, const void *z_uncond,
+                                   void *delta, float gamma, size_t n, void *z_uncond_out,
+                                   void *guided_out, void *stream);
+
+/* Component entry points: the kernels the steps run, on caller buffers
+ * (device pointers only), for parity tests and for callers composing their
+ * own pipeline. */
+
+/* y = a W^T + bias with a fused epilogue, a [M, K], W [N, K] (row-major,
+ * dtype), bias [N] (dtype, may be NULL). bf16 runs on the tcgen05 tensor cores
+ * (K % 64 == 0, N % 128 == 0); f32 on CUDA cores (K % 4 == 0, N % 4 == 0).
+ *   LAZYMAR_EPI_BIAS     out [M, ldo] dtype = y
+ *   LAZYMAR_EPI_GELU     out [M, ldo] dtype = GELU(y) (erf form)
+ *   LAZYMAR_EPI_RESIDUAL out [M, ldo] fp32 += y
+ *   LAZYMAR_EPI_QKV      N = 3D: columns 0..D-1 -> out [M, D]; D..2D-1 ->
+ *                        k_out[row_map[m], :]; 2D..3D-1 -> v_out[row_map[m], :]
+ *                        (row_map NULL = identity; the cache scatter of Eq. 9)
+ * flags: 0 automatic tile width, 1 force 128, 2 force 256 (bf16). */
+enum { LAZYMAR_EPI_BIAS = 0, LAZYMAR_EPI_GELU = 1, LAZYMAR_EPI_RESIDUAL = 2, LAZYMAR_EPI_QKV = 3 };
+lazymar_status lazymar_linear(int dtype, int epilogue, const void *a, const void *w,
+                              const void *bias, int M, int N, int K, void *out, int ldo,
+                              void *k_out, void *v_out, const int32_t *row_map, int flags,
+                              void *stream);
+
+/* Multi-head bidirectional attention of Eq. 3 with a query subset: for each row
+ * r and head h, O[r, j] = softmax(Q[r, j] K[r]^T / sqrt(dh)) V[r] over all T
+ * keys. q, o: [rows, n_q, heads*head_dim]; k, v: [rows, T, heads*head_dim]
+ * (dtype). bf16: head_dim 64 or 80, mma tensor cores with TMA-staged K/V. */
+lazymar_status lazymar_attention(int dtype, const void *q, const void *k, const void *v, void *o,
+                                 int rows, int n_q, int T, int heads, int head_dim, void *stream);
+
+/* LayerNorm over D of fp32 rows: y[m] = LN(x[row_map ? row_map[m] : m]) * g + b,
+ * y in dtype, g/b in dtype. D % 128 == 0, D <= 2048. */
+lazymar_status lazymar_layernorm(int dtype, const float *x, const int32_t *row_map, const void *g,
+                                 const void *b, void *y, int M, int D, float eps, void *stream);
+
+/* Schedule of periodic cache-reuse-refreshment (host only, no GPU): steps
+ * k < k0 are full, then full whenever (k - k0) % tau == 0; other steps are
+ * cached and reuse the condition cache when use_cond_cache and tau_cfg > 0 and
+ * (k - k0) % tau_cfg != 0. Returns bit 0 = full step, bit 1 = reuse the
+ * condition cache, or -1 for invalid arguments. */
+int lazymar_plan_step(int k, int k0, int tau, int tau_cfg, int use_cond_cache);
+
+/* Waits for `stream`, then reports (and clears) errors the handle's kernels
+ * latched on the device: TIMEOUT, DEVICE, or CUDA for an asynchronous fault. */
+lazymar_status lazymar_sync(lazymar_handle *h, void *stream);
+
+/* As lazymar_sync for the component entry points of the current device. */
+lazymar_status lazymar_device_check(void *stream);
+
+/* Per kernel class: launches, algorithmic flops and bytes, and (while
+ * profiling is on) device time from CUDA events recorded around each launch on
+ * its stream. lazymar_get_stats waits for the recorded events. */
+enum {
+  LAZYMAR_K_GEMM = 0, LAZYMAR_K_ATTENTION = 1, LAZYMAR_K_LAYERNORM = 2, LAZYMAR_K_SELECT = 3,
+  LAZYMAR_K_EMBED = 4, LAZYMAR_K_CFG = 5, LAZYMAR_K_OTHER = 6, LAZYMAR_K_COUNT = 7
+};
+typedef struct lazymar_kernel_stats {
+  long long launches;
+  long long timed_launches;
+  double ms;
+  double flops;
+  double bytes;
+} lazymar_kernel_stats;
+typedef struct lazymar_stats {
+  lazymar_kernel_stats k[LAZYMAR_K_COUNT];
+} lazymar_stats;
+lazymar_status lazymar_set_profiling(lazymar_handle *h, int enable);
+lazymar_status lazymar_get_stats(lazymar_handle *h, lazymar_stats *out);
+lazymar_status lazymar_reset_stats(lazymar_handle *h);
+
+const char *lazymar_status_string(lazymar_status s);
+/* Text of the last error on the calling thread (empty if none). */
+const char *lazymar_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* LAZYMAR_H */

@@ -1,0 +1,369 @@
+// GEMMs of the MAR block: QKV, attention output, MLP up and down projections
+// (Eq. 9's F(X[I_compute]) for the token subset, and the full-layer forms).
+//
+// bf16: a persistent, warp-specialised tcgen05 kernel. Warp 0 streams A and W
+// tiles with TMA (128B swizzle) into a ring of shared-memory stages, warp 1
+// issues tcgen05.mma (128 x BN x 16, fp32 accumulators in tensor memory,
+// double-buffered so the epilogue of one tile overlaps the main loop of the
+// next) and eight epilogue warps drain the accumulators with tcgen05.ld and
+// apply the fused epilogue: bias, GELU, fp32 residual add, or the Q/K/V split
+// with the K/V rows scattered into the token cache (row_map).
+//
+// f32: a 64x64 register-tiled CUDA-core kernel with the same epilogues (the
+// tensor cores have no fp32 kind; this serves the fp32 configuration).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "lazymar_internal.cuh"
+
+namespace lm {
+
+// ---------------------------------------------------------------------------
+// Epilogue shared by both kernels: NC consecutive columns of one row.
+// ---------------------------------------------------------------------------
+template <typename T, int NC>
+__device__ __forceinline__ void epilogue_apply(const GemmEpi& e, int row, int col0, float* v) {
+  if (e.bias) {
+    float bv[NC];
+    Vec<T, NC>::load(static_cast<const T*>(e.bias) + col0, bv);
+#pragma unroll
+    for (int i = 0; i < NC; ++i) v[i] += bv[i];
+  }
+  switch (e.mode) {
+    case LAZYMAR_EPI_GELU:
+#pragma unroll
+      for (int i = 0; i < NC; ++i) v[i] = gelu_erf(v[i]);
+      Vec<T, NC>::store(static_cast<T*>(e.out) + (size_t)row * e.ldo + col0, v);
+      break;
+    case LAZYMAR_EPI_RESIDUAL: {
+      float* o = static_cast<float*>(e.out) + (size_t)row * e.ldo + col0;
+      float r[NC];
+      Vec<float, NC>::load(o, r);
+#pragma unroll
+      for (int i = 0; i < NC; ++i) r[i] += v[i];
+      Vec<float, NC>::store(o, r);
+      break;
+    }
+    case LAZYMAR_EPI_QKV: {
+      const int part = col0 / e.D;
+      const int c = col0 - part * e.D;
+      T* dst;
+      if (part == 0) {
+        dst = static_cast<T*>(e.out) + (size_t)row * e.D + c;
+      } else {
+        const int drow = e.row_map ? e.row_map[row] : row;
+        dst = static_cast<T*>(part == 1 ? e.k_out : e.v_out) + (size_t)drow * e.D + c;
+      }
+      Vec<T, NC>::store(dst, v);
+      break;
+    }
+    default:
+      Vec<T, NC>::store(static_cast<T*>(e.out) + (size_t)row * e.ldo + col0, v);
+      break;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// tcgen05 kernel
+// ---------------------------------------------------------------------------
+namespace tc {
+constexpr int BM = 128;  // rows per tile = MMA M (one accumulator lane per row)
+constexpr int BK = 64;   // one 128-byte swizzle atom of bf16 along K
+constexpr int kEpiWarps = 8;
+constexpr int kThreads = 64 + kEpiWarps * 32;
+
+template <int BN>
+struct Cfg {
+  static constexpr int STAGES = (BN == 256) ? 4 : 6;
+  static constexpr uint32_t A_BYTES = BM * BK * 2;
+  static constexpr uint32_t B_BYTES = BN * BK * 2;
+  static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulator buffers
+  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + 256;
+  // Instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1),
+  // B bf16 (bits 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
+  static constexpr uint32_t IDESC =
+      (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+};
+
+// Shared-memory matrix descriptor of a K-major tile written by TMA with
+// SWIZZLE_128B: rows of 128 bytes, 8-row groups 1024 bytes apart (stride byte
+// offset), descriptor version 1 (bit 46), layout SWIZZLE_128B (2 at bit 61).
+// The leading byte offset is not used by this layout.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+         ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+}  // namespace tc
+
+template <int BN>
+__global__ void __launch_bounds__(tc::kThreads, 1)
+    gemm_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M,
+                        int N, int K, GemmEpi epi, unsigned* err) {
+  using C = tc::Cfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + C::STAGES * C::A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  uint64_t* empty = full + C::STAGES;
+  uint64_t* acc_full = empty + C::STAGES;
+  uint64_t* acc_empty = acc_full + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int num_m = (M + tc::BM - 1) / tc::BM;
+  const int tiles = num_m * (N / BN);
+  const int KB = K / tc::BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], tc::kEpiWarps);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tmA);
+    prefetch_tmap(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
+        const int m0 = (tile % num_m) * tc::BM, n0 = (tile / num_m) * BN;
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
+          mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
+          tma_load_2d(&tmA, &full[stage], sA + stage * C::A_BYTES, kb * tc::BK, m0);
+          tma_load_2d(&tmB, &full[stage], sB + stage * C::B_BYTES, kb * tc::BK, n0);
+          if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int it = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x, ++it) {
+        const int buf = it & 1;
+        const uint32_t use = (uint32_t)(it >> 1) & 1u;
+        if (!mbar_wait(&acc_empty[buf], use ^ 1u, abort_flag, err)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag, err)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t a0 = tc::sw128_desc(smem_u32(sA + stage * C::A_BYTES));
+          const uint64_t b0 = tc::sw128_desc(smem_u32(sB + stage * C::B_BYTES));
+#pragma unroll
+          for (int k = 0; k < tc::BK / 16; ++k)  // +32 bytes per K=16 step inside the swizzle atom
+            umma_bf16(d_tmem, a0 + 2 * k, b0 + 2 * k, C::IDESC, (kb | k) != 0 ? 1u : 0u);
+          umma_commit(&empty[stage]);
+          if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
+        }
+        if (ok) umma_commit(&acc_full[buf]);
+      }
+    }
+    __syncwarp();
+  } else {
+    // ---------------- epilogue warps ----------------
+    const int ew = warp - 2;        // 0..7
+    const int quarter = warp & 3;   // tensor-memory lanes this warp may read
+    const int half = ew >> 2;       // which half of the tile's columns
+    constexpr int CHUNKS = BN / 64; // 32-column chunks per half
+    int it = 0;
+    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++it) {
+      const int buf = it & 1;
+      const uint32_t use = (uint32_t)(it >> 1) & 1u;
+      const bool ok = mbar_wait(&acc_full[buf], use, abort_flag, err);
+      if (__any_sync(0xffffffffu, !ok)) break;
+      tc_fence_after();
+      const int m0 = (tile % num_m) * tc::BM, n0 = (tile / num_m) * BN;
+      const int row = m0 + quarter * 32 + lane;
+#pragma unroll 1
+      for (int c = half * CHUNKS; c < (half + 1) * CHUNKS; ++c) {
+        uint32_t r[32];
+        tmem_ld32(tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN + c * 32), r);
+        tmem_wait_ld();
+        if (row < M) {
+          float v[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+          epilogue_apply<bf16, 32>(epi, row, n0 + c * 32, v);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[buf]);
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// fp32 CUDA-core kernel: 64 x 64 tile, 256 threads, 4 x 4 outputs per thread
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) gemm_f32_kernel(const float* __restrict__ A, const float* __restrict__ W, int M,
+                                                       int N, int K, GemmEpi epi) {
+  __shared__ float As[16][64 + 4];
+  __shared__ float Ws[16][64 + 4];
+  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+  const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
+  float acc[4][4] = {};
+  for (int k0 = 0; k0 < K; k0 += 16) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int idx = threadIdx.x + i * 256;
+      const int r = idx >> 4, c = idx & 15;
+      As[c][r] = (m0 + r < M && k0 + c < K) ? A[(size_t)(m0 + r) * K + k0 + c] : 0.f;
+      Ws[c][r] = (n0 + r < N && k0 + c < K) ? W[(size_t)(n0 + r) * K + k0 + c] : 0.f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < 16; ++kk) {
+      float a[4], b[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        a[i] = As[kk][ty * 4 + i];
+        b[i] = Ws[kk][tx * 4 + i];
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+  const int col = n0 + tx * 4;
+  if (col >= N) return;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int row = m0 + ty * 4 + i;
+    if (row < M) epilogue_apply<float, 4>(epi, row, col, acc[i]);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------
+static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor map over a row-major [outer, inner] matrix with the given
+// row pitch, box [box_outer, box_inner], out-of-bounds elements read as zero.
+bool make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t pitch_bytes,
+                    uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swz) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {pitch_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t es[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool gemm_supported(int dtype, int M, int N, int K, const GemmEpi& epi, const char** why) {
+  if (M < 0 || N <= 0 || K <= 0) { *why = "M >= 0, N > 0, K > 0 required"; return false; }
+  if (epi.mode == LAZYMAR_EPI_QKV && (epi.D <= 0 || N != 3 * epi.D)) { *why = "QKV epilogue needs N = 3D"; return false; }
+  if (dtype == LAZYMAR_BF16) {
+    if (K % 64 != 0) { *why = "bf16 GEMM needs K % 64 == 0"; return false; }
+    if (N % 128 != 0) { *why = "bf16 GEMM needs N % 128 == 0"; return false; }
+    if (epi.mode == LAZYMAR_EPI_QKV && epi.D % 32 != 0) { *why = "QKV epilogue needs D % 32 == 0"; return false; }
+    if (epi.mode != LAZYMAR_EPI_QKV && epi.ldo % 8 != 0) { *why = "ldo % 8 == 0 required"; return false; }
+  } else if (dtype == LAZYMAR_F32) {
+    if (K % 4 != 0 || N % 4 != 0) { *why = "f32 GEMM needs K % 4 == 0 and N % 4 == 0"; return false; }
+    if (epi.mode == LAZYMAR_EPI_QKV && epi.D % 4 != 0) { *why = "QKV epilogue needs D % 4 == 0"; return false; }
+    if (epi.mode != LAZYMAR_EPI_QKV && epi.ldo % 4 != 0) { *why = "ldo % 4 == 0 required"; return false; }
+  } else {
+    *why = "unknown dtype";
+    return false;
+  }
+  return true;
+}
+
+template <int BN>
+static cudaError_t launch_tc(const Ctx& c, const void* A, const void* W, int M, int N, int K, const GemmEpi& epi) {
+  using C = tc::Cfg<BN>;
+  CUtensorMap ta, tb;
+  if (!make_tmap_bf16(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * 2, tc::BK, tc::BM,
+                      CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_tmap_bf16(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, tc::BK, BN, CU_TENSOR_MAP_SWIZZLE_128B))
+    return cudaErrorInvalidValue;
+  static int attr_set[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)C::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set[dev] = 1;
+  }
+  const int tiles = ((M + tc::BM - 1) / tc::BM) * (N / BN);
+  const int grid = tiles < c.num_sms ? tiles : c.num_sms;
+  gemm_bf16_tc_kernel<BN><<<grid, tc::kThreads, C::SMEM, c.stream>>>(ta, tb, M, N, K, epi, c.err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, int M, int N, int K,
+                        const GemmEpi& epi, int flags) {
+  if (M == 0) return cudaSuccess;
+  if (dtype == LAZYMAR_F32) {
+    dim3 grid((N + 63) / 64, (M + 63) / 64);
+    gemm_f32_kernel<<<grid, 256, 0, c.stream>>>(static_cast<const float*>(A), static_cast<const float*>(W), M, N,
+                                                 K, epi);
+    return cudaGetLastError();
+  }
+  // Tile width: the one with fewer tile-waves x tile-time over the SMs.
+  int bn = 128;
+  if (flags == 2 && N % 256 == 0) {
+    bn = 256;
+  } else if (flags == 0 && N % 256 == 0) {
+    const long mt = (M + tc::BM - 1) / tc::BM;
+    const long w128 = (mt * (N / 128) + c.num_sms - 1) / c.num_sms * 128;
+    const long w256 = (mt * (N / 256) + c.num_sms - 1) / c.num_sms * 256;
+    if (w256 <= w128) bn = 256;
+  }
+  return bn == 256 ? launch_tc<256>(c, A, W, M, N, K, epi) : launch_tc<128>(c, A, W, M, N, K, epi);
+}
+
+}  // namespace lm

@@ -1,0 +1,290 @@
+// Row-wise and elementwise kernels of the decoding step:
+//   - embedding of the input tokens (Eq. 6): class embedding / zero fake
+//     conditional tokens on the buffer positions, latent projection or mask
+//     embedding on the image positions, plus the position embedding;
+//   - LayerNorm of fp32 residual rows into the GEMM operand dtype, optionally
+//     gathering rows (the step's switch from all tokens to I_compute) and
+//     keeping an fp32 copy of the gathered rows as the compact residual stream;
+//   - the final LayerNorm that scatters the recomputed rows into the output
+//     cache (Eq. 9: outputs of I_cache tokens stay as cached);
+//   - classifier-free guidance with the condition cache (Eq. 7, Eq. 10) on
+//     16-byte vectors.
+// All of these are bound by HBM bandwidth; one warp per row (LayerNorm) or
+// grid-stride 16-byte vectors (CFG) keeps loads coalesced.
+#include "lazymar_internal.cuh"
+
+namespace lm {
+
+// ---------------------------------------------------------------------------
+// Embedding
+// ---------------------------------------------------------------------------
+template <typename TW>
+__global__ void __launch_bounds__(256) embed_kernel(const float* __restrict__ lat, const uint8_t* __restrict__ mask,
+                                                    const int* __restrict__ labels, const TW* __restrict__ pos,
+                                                    const TW* __restrict__ cls, const TW* __restrict__ memb,
+                                                    const TW* __restrict__ ew, const TW* __restrict__ eb,
+                                                    float* __restrict__ H, int B, int T, int nb, int n_img, int D,
+                                                    int tdim, int n_classes, unsigned* err) {
+  __shared__ float sl[64];
+  const int tok = blockIdx.x;  // r * T + t
+  const int r = tok / T, t = tok - r * T;
+  const bool cond = r < B;
+  const int pair = cond ? r : r - B;
+  float* out = H + (size_t)tok * D;
+  const TW* p = pos + (size_t)t * D;
+  if (t < nb) {
+    const TW* c = nullptr;
+    if (cond) {
+      int y = labels[pair];
+      if (y < 0 || y >= n_classes) {
+        if (threadIdx.x == 0) atomicOr(err, ERR_LABEL);
+        y = 0;
+      }
+      c = cls + (size_t)y * D;
+    }
+    for (int d = threadIdx.x; d < D; d += blockDim.x) out[d] = to_f(p[d]) + (c ? to_f(c[d]) : 0.f);
+    return;
+  }
+  const int i = t - nb;
+  if (mask[(size_t)pair * n_img + i]) {
+    for (int d = threadIdx.x; d < D; d += blockDim.x) out[d] = to_f(p[d]) + to_f(memb[d]);
+    return;
+  }
+  const float* lr = lat + ((size_t)pair * n_img + i) * tdim;
+  for (int j = threadIdx.x; j < tdim; j += blockDim.x) sl[j] = lr[j];
+  __syncthreads();
+  for (int d = threadIdx.x; d < D; d += blockDim.x) {
+    const TW* w = ew + (size_t)d * tdim;
+    float acc = to_f(eb[d]);
+    for (int j = 0; j < tdim; ++j) acc = fmaf(to_f(w[j]), sl[j], acc);
+    out[d] = to_f(p[d]) + acc;
+  }
+}
+
+cudaError_t launch_embed(const Ctx& c, int dtype, const float* lat, const uint8_t* mask, const int* labels,
+                         const void* pos, const void* cls, const void* memb, const void* ew, const void* eb, float* H,
+                         int rows, int B, int T, int nb, int n_img, int D, int tdim, int n_classes) {
+  if (rows == 0) return cudaSuccess;
+  const unsigned grid = (unsigned)(rows * T);
+  if (dtype == LAZYMAR_BF16)
+    embed_kernel<bf16><<<grid, 256, 0, c.stream>>>(lat, mask, labels, (const bf16*)pos, (const bf16*)cls,
+                                                   (const bf16*)memb, (const bf16*)ew, (const bf16*)eb, H, B, T, nb,
+                                                   n_img, D, tdim, n_classes, c.err);
+  else
+    embed_kernel<float><<<grid, 256, 0, c.stream>>>(lat, mask, labels, (const float*)pos, (const float*)cls,
+                                                    (const float*)memb, (const float*)ew, (const float*)eb, H, B, T,
+                                                    nb, n_img, D, tdim, n_classes, c.err);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// LayerNorm (one warp per row, NV float4 per lane: D = 128 * NV)
+// ---------------------------------------------------------------------------
+template <int NV>
+__device__ __forceinline__ void ln_stats(const float4 (&v)[NV], int D, float eps, float& mean, float& rstd) {
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) s += (v[i].x + v[i].y) + (v[i].z + v[i].w);
+  mean = warp_sum(s) / (float)D;
+  float q = 0.f;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    const float a = v[i].x - mean, b = v[i].y - mean, cc = v[i].z - mean, d = v[i].w - mean;
+    q += (a * a + b * b) + (cc * cc + d * d);
+  }
+  rstd = rsqrtf(warp_sum(q) / (float)D + eps);
+}
+
+template <typename TO>
+__device__ __forceinline__ void ln_write4(TO* y, const TO* g, const TO* b, int col, float4 x, float mean, float rstd) {
+  float o[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+  for (int k = 0; k < 4; ++k) o[k] = (o[k] - mean) * rstd * to_f(g[col + k]) + to_f(b[col + k]);
+  if constexpr (sizeof(TO) == 2) {
+    __nv_bfloat162 h0 = __floats2bfloat162_rn(o[0], o[1]), h1 = __floats2bfloat162_rn(o[2], o[3]);
+    uint2 u;
+    u.x = *reinterpret_cast<uint32_t*>(&h0);
+    u.y = *reinterpret_cast<uint32_t*>(&h1);
+    *reinterpret_cast<uint2*>(y + col) = u;
+  } else {
+    *reinterpret_cast<float4*>(y + col) = make_float4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+template <typename TO, int NV>
+__global__ void __launch_bounds__(256) layernorm_kernel(const float* __restrict__ x, const int* __restrict__ row_map,
+                                                        const TO* __restrict__ g, const TO* __restrict__ b,
+                                                        TO* __restrict__ y, float* __restrict__ x_copy, int M, int D,
+                                                        float eps) {
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (row >= M) return;
+  const int src = row_map ? row_map[row] : row;
+  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)src * D);
+  float4 v[NV];
+#pragma unroll
+  for (int i = 0; i < NV; ++i) v[i] = xr[lane + 32 * i];
+  if (x_copy) {
+    float4* cr = reinterpret_cast<float4*>(x_copy + (size_t)row * D);
+#pragma unroll
+    for (int i = 0; i < NV; ++i) cr[lane + 32 * i] = v[i];
+  }
+  float mean, rstd;
+  ln_stats<NV>(v, D, eps, mean, rstd);
+  TO* yr = y + (size_t)row * D;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) ln_write4<TO>(yr, g, b, 4 * (lane + 32 * i), v[i], mean, rstd);
+}
+
+template <typename TO, int NV>
+__global__ void __launch_bounds__(256) final_ln_kernel(const float* __restrict__ x, const int* __restrict__ row_map,
+                                                       int T, int nb, int n_img, const TO* __restrict__ g,
+                                                       const TO* __restrict__ b, TO* __restrict__ z, int M, int D,
+                                                       float eps) {
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (row >= M) return;
+  const int tok = row_map ? row_map[row] : row;
+  const int r = tok / T, t = tok - r * T;
+  if (t < nb) return;
+  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)row * D);
+  float4 v[NV];
+#pragma unroll
+  for (int i = 0; i < NV; ++i) v[i] = xr[lane + 32 * i];
+  float mean, rstd;
+  ln_stats<NV>(v, D, eps, mean, rstd);
+  TO* zr = z + ((size_t)r * n_img + (t - nb)) * D;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) ln_write4<TO>(zr, g, b, 4 * (lane + 32 * i), v[i], mean, rstd);
+}
+
+#define LM_LN_DISPATCH(KERNEL, TO, ...)                                                    \
+  switch (D / 128) {                                                                     \
+    case 1: KERNEL<TO, 1><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;               \
+    case 2: KERNEL<TO, 2><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;               \
+    case 4: KERNEL<TO, 4><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;               \
+    case 6: KERNEL<TO, 6><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;               \
+    case 8: KERNEL<TO, 8><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;               \
+    case 10: KERNEL<TO, 10><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;             \
+    case 12: KERNEL<TO, 12><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;             \
+    case 16: KERNEL<TO, 16><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;             \
+    default: return cudaErrorInvalidValue;                                               \
+  }
+
+bool layernorm_width_ok(int D) {
+  const int k = D / 128;
+  return D % 128 == 0 && (k == 1 || k == 2 || k == 4 || k == 6 || k == 8 || k == 10 || k == 12 || k == 16);
+}
+
+cudaError_t launch_layernorm(const Ctx& c, int dtype, const float* x, const int* row_map, const void* g,
+                             const void* b, void* y, float* x_copy, int M, int D, float eps) {
+  if (M == 0) return cudaSuccess;
+  const unsigned grid = (unsigned)((M + 7) / 8);
+  if (dtype == LAZYMAR_BF16) {
+    LM_LN_DISPATCH(layernorm_kernel, bf16, x, row_map, (const bf16*)g, (const bf16*)b, (bf16*)y, x_copy, M, D, eps)
+  } else {
+    LM_LN_DISPATCH(layernorm_kernel, float, x, row_map, (const float*)g, (const float*)b, (float*)y, x_copy, M, D,
+                   eps)
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_final_ln(const Ctx& c, int dtype, const float* x, const int* row_map, int T, int nb, int n_img,
+                            const void* g, const void* b, void* z, int M, int D, float eps) {
+  if (M == 0) return cudaSuccess;
+  const unsigned grid = (unsigned)((M + 7) / 8);
+  if (dtype == LAZYMAR_BF16) {
+    LM_LN_DISPATCH(final_ln_kernel, bf16, x, row_map, T, nb, n_img, (const bf16*)g, (const bf16*)b, (bf16*)z, M, D,
+                   eps)
+  } else {
+    LM_LN_DISPATCH(final_ln_kernel, float, x, row_map, T, nb, n_img, (const float*)g, (const float*)b, (float*)z, M,
+                   D, eps)
+  }
+  return cudaGetLastError();
+}
+
+// fp32 -> dtype copy (the block output features used as the selection
+// criterion when criterion == FEATURE).
+template <typename TO>
+__global__ void cast_kernel(const float* __restrict__ x, TO* __restrict__ y, size_t n) {
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x)
+    y[i] = from_f<TO>(x[i]);
+}
+cudaError_t launch_cast(const Ctx& c, int dtype, const float* x, void* y, size_t n) {
+  if (n == 0) return cudaSuccess;
+  const unsigned grid = (unsigned)((n + 255) / 256 < (size_t)c.num_sms * 8 ? (n + 255) / 256 : (size_t)c.num_sms * 8);
+  if (dtype == LAZYMAR_BF16)
+    cast_kernel<bf16><<<grid, 256, 0, c.stream>>>(x, (bf16*)y, n);
+  else
+    cast_kernel<float><<<grid, 256, 0, c.stream>>>(x, (float*)y, n);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Classifier-free guidance with the condition cache
+// ---------------------------------------------------------------------------
+template <typename T>
+__device__ __forceinline__ void cfg_elems(int mode, float gamma, const float* c, const float* u_in, float* d, float* u,
+                                          float* g, int n) {
+  for (int i = 0; i < n; ++i) {
+    float uu;
+    if (mode == LAZYMAR_CFG_REUSE) {
+      uu = c[i] - d[i];
+    } else {
+      uu = u_in[i];
+      if (mode == LAZYMAR_CFG_REFRESH) d[i] = c[i] - uu;
+    }
+    u[i] = uu;
+    g[i] = uu + gamma * (c[i] - uu);
+  }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) cfg_kernel(int mode, const T* __restrict__ zc, const T* __restrict__ zu,
+                                                  T* __restrict__ delta, float gamma, size_t n, T* __restrict__ zu_out,
+                                                  T* __restrict__ g_out) {
+  constexpr int V = 16 / sizeof(T);
+  const size_t nv = n / V;
+  const size_t stride = (size_t)gridDim.x * blockDim.x;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < nv; i += stride) {
+    const size_t o = i * V;
+    float c[V], u[V], d[V], uo[V], g[V];
+    Vec<T, V>::load(zc + o, c);
+    if (mode == LAZYMAR_CFG_REUSE) Vec<T, V>::load(delta + o, d);
+    else Vec<T, V>::load(zu + o, u);
+    cfg_elems<T>(mode, gamma, c, u, d, uo, g, V);
+    if (mode == LAZYMAR_CFG_REFRESH) Vec<T, V>::store(delta + o, d);
+    if (mode == LAZYMAR_CFG_REUSE && zu_out) Vec<T, V>::store(zu_out + o, uo);
+    if (g_out) Vec<T, V>::store(g_out + o, g);
+  }
+  // scalar tail
+  const size_t tail0 = nv * V;
+  const size_t gt = blockIdx.x * (size_t)blockDim.x + threadIdx.x;
+  if (gt < n - tail0) {
+    const size_t o = tail0 + gt;
+    float c = to_f(zc[o]), u = 0.f, d = 0.f, uo, g;
+    if (mode == LAZYMAR_CFG_REUSE) d = to_f(delta[o]);
+    else u = to_f(zu[o]);
+    cfg_elems<T>(mode, gamma, &c, &u, &d, &uo, &g, 1);
+    if (mode == LAZYMAR_CFG_REFRESH) delta[o] = from_f<T>(d);
+    if (mode == LAZYMAR_CFG_REUSE && zu_out) zu_out[o] = from_f<T>(uo);
+    if (g_out) g_out[o] = from_f<T>(g);
+  }
+}
+
+cudaError_t launch_cfg(const Ctx& c, int dtype, int mode, const void* zc, const void* zu, void* delta, float gamma,
+                       size_t n, void* zu_out, void* g_out) {
+  if (n == 0) return cudaSuccess;
+  const size_t V = dtype == LAZYMAR_BF16 ? 8 : 4;
+  size_t blocks = (n / V + 255) / 256;
+  const size_t cap = (size_t)c.num_sms * 8;
+  if (blocks > cap) blocks = cap;
+  if (blocks == 0) blocks = 1;
+  if (dtype == LAZYMAR_BF16)
+    cfg_kernel<bf16><<<(unsigned)blocks, 256, 0, c.stream>>>(mode, (const bf16*)zc, (const bf16*)zu, (bf16*)delta,
+                                                             gamma, n, (bf16*)zu_out, (bf16*)g_out);
+  else
+    cfg_kernel<float><<<(unsigned)blocks, 256, 0, c.stream>>>(mode, (const float*)zc, (const float*)zu,
+                                                              (float*)delta, gamma, n, (float*)zu_out, (float*)g_out);
+  return cudaGetLastError();
+}
+
+}  // namespace lm

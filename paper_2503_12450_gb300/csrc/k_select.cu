@@ -1,0 +1,161 @@
+// Token selection of Eq. 8.
+//
+// similarity_kernel: one warp per token, spread over the whole GPU (a row has
+// only T tokens, so one CTA per row would leave most SMs idle while streaming
+// 2 x rows x T x D elements). Each lane reads 16-byte vectors of the current
+// and cached representation and accumulates the dot product and both squared
+// norms in fp64. bf16 x bf16 products are exact in fp64, and so are their sums
+// for any realistic dynamic range, which makes S independent of the summation
+// order: the oracle's fp64 sum gives bit-identical S, hence bit-identical
+// selections. The current vector is copied over the cached one (the cache now
+// holds this step's values).
+//
+// topk_kernel: one CTA per row. Each token's rank under the strict total order
+// (S ascending, index ascending; NaN counted as -inf) is counted against all T
+// similarities held in shared memory; tokens with rank < N are I_compute. A
+// block-wide ballot/prefix scan writes them in ascending index order together
+// with the gather/scatter row map r*T + t.
+#include <cfloat>
+
+#include "lazymar_internal.cuh"
+
+namespace lm {
+
+template <typename T>
+__global__ void __launch_bounds__(256) similarity_kernel(const T* __restrict__ cur, T* __restrict__ cache,
+                                                         double* __restrict__ S, long long ntok, int D, int copy) {
+  constexpr int V = 16 / sizeof(T);
+  const long long tok = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (tok >= ntok) return;
+  const T* a = cur + tok * D;
+  T* c = cache + tok * D;
+  double dot = 0.0, na = 0.0, nc = 0.0;
+  for (int i = lane * V; i < D; i += 32 * V) {
+    float av[V], cv[V];
+    Vec<T, V>::load(a + i, av);
+    Vec<T, V>::load(c + i, cv);
+#pragma unroll
+    for (int k = 0; k < V; ++k) {
+      const double x = (double)av[k], y = (double)cv[k];
+      dot = fma(x, y, dot);
+      na = fma(x, x, na);
+      nc = fma(y, y, nc);
+    }
+    if (copy) *reinterpret_cast<uint4*>(c + i) = *reinterpret_cast<const uint4*>(a + i);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    dot += __shfl_xor_sync(0xffffffffu, dot, o);
+    na += __shfl_xor_sync(0xffffffffu, na, o);
+    nc += __shfl_xor_sync(0xffffffffu, nc, o);
+  }
+  if (lane == 0) {
+    const double eps = 1e-8;
+    S[tok] = dot / sqrt(fmax(na * nc, eps * eps));
+  }
+}
+
+cudaError_t launch_similarity(const Ctx& c, int dtype, const void* cur, void* cache, double* S, int rows, int T, int D,
+                              bool copy) {
+  const long long ntok = (long long)rows * T;
+  if (ntok == 0) return cudaSuccess;
+  const unsigned grid = (unsigned)((ntok + 7) / 8);
+  if (dtype == LAZYMAR_BF16)
+    similarity_kernel<bf16><<<grid, 256, 0, c.stream>>>((const bf16*)cur, (bf16*)cache, S, ntok, D, copy ? 1 : 0);
+  else
+    similarity_kernel<float><<<grid, 256, 0, c.stream>>>((const float*)cur, (float*)cache, S, ntok, D, copy ? 1 : 0);
+  return cudaGetLastError();
+}
+
+constexpr int kTopkThreads = 512;
+
+__global__ void __launch_bounds__(kTopkThreads) topk_kernel(const double* __restrict__ S, int T, int N,
+                                                            int* __restrict__ idx, int* __restrict__ row_map) {
+  extern __shared__ double sS[];  // T keys
+  __shared__ int s_wcount[kTopkThreads / 32];
+  __shared__ int s_woff[kTopkThreads / 32];
+  __shared__ int s_total;
+  unsigned char* sel = reinterpret_cast<unsigned char*>(sS + T);
+  const int r = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int t = tid; t < T; t += kTopkThreads) {
+    const double s = S[(size_t)r * T + t];
+    sS[t] = (s != s) ? -DBL_MAX * 2.0 : s;  // NaN -> -inf
+  }
+  __syncthreads();
+  for (int t = tid; t < T; t += kTopkThreads) {
+    const double st = sS[t];
+    int rank = 0;
+    for (int u = 0; u < T; ++u) {
+      const double su = sS[u];
+      rank += (su < st) || (su == st && u < t);
+    }
+    sel[t] = rank < N;
+  }
+  __syncthreads();
+  int base = 0;
+  for (int c0 = 0; c0 < T; c0 += kTopkThreads) {
+    const int t = c0 + tid;
+    const bool f = t < T && sel[t];
+    const unsigned bal = __ballot_sync(0xffffffffu, f);
+    if (lane == 0) s_wcount[warp] = __popc(bal);
+    __syncthreads();
+    if (warp == 0) {
+      const int v = lane < kTopkThreads / 32 ? s_wcount[lane] : 0;
+      int incl = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int n = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += n;
+      }
+      if (lane < kTopkThreads / 32) s_woff[lane] = incl - v;
+      if (lane == 31) s_total = incl;
+    }
+    __syncthreads();
+    if (f) {
+      const int pos = base + s_woff[warp] + __popc(bal & ((1u << lane) - 1u));
+      idx[(size_t)r * N + pos] = t;
+      if (row_map) row_map[(size_t)r * N + pos] = r * T + t;
+    }
+    base += s_total;
+    __syncthreads();
+  }
+}
+
+cudaError_t launch_topk(const Ctx& c, const double* S, int rows, int T, int N, int* idx, int* row_map) {
+  if (rows == 0 || N == 0) return cudaSuccess;
+  const size_t smem = (size_t)T * sizeof(double) + (size_t)T;
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  topk_kernel<<<rows, kTopkThreads, smem, c.stream>>>(S, T, N, idx, row_map);
+  return cudaGetLastError();
+}
+
+// Caller-chosen I_compute: copied after checking range and strict increase per
+// row; a violation is latched as ERR_INDEX and the index is clamped into
+// [0, T) so that no later gather or scatter leaves the row.
+__global__ void idx_check_kernel(const int* __restrict__ in, int rows, int T, int N, int* __restrict__ idx,
+                                 int* __restrict__ row_map, unsigned* err) {
+  const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+  if (i >= (long long)rows * N) return;
+  const int r = (int)(i / N), j = (int)(i - (long long)r * N);
+  int v = in[i];
+  bool ok = v >= 0 && v < T && (j == 0 || in[i - 1] < v);
+  if (!ok) {
+    atomicOr(err, ERR_INDEX);
+    v = v < 0 ? 0 : (v >= T ? T - 1 : v);
+  }
+  idx[i] = v;
+  row_map[i] = r * T + v;
+}
+
+cudaError_t launch_idx_check(const Ctx& c, const int* in, int rows, int T, int N, int* idx, int* row_map) {
+  const long long n = (long long)rows * N;
+  if (n == 0) return cudaSuccess;
+  idx_check_kernel<<<(unsigned)((n + 255) / 256), 256, 0, c.stream>>>(in, rows, T, N, idx, row_map, c.err);
+  return cudaGetLastError();
+}
+
+}  // namespace lm

@@ -17,4 +17,7 @@ from .inputs import (  # noqa: F401
     step_state,
     tiny_state,
     n_compute,
+    tensor,
+    similarity_inputs,
+    distinct_rows,
 )

@@ -174,3 +174,37 @@ def step_state(cfg, order, table, n_decoded):
 def tiny_state(cfg, order, table, before=24, after=32):
     """The tiny workload: a forward with 24 decoded tokens, then one with 8 more."""
     return step_state(cfg, order, table, before), step_state(cfg, order, table, after)
+
+
+def tensor(shape, seed, std=1.0, dtype="fp32", mean=0.0):
+    """Seeded N(mean, std^2) fp32 tensor; bf16-representable when dtype == 'bf16'."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    x = (rng.standard_normal(shape, dtype=np.float32) * np.float32(std) + np.float32(mean)).astype(np.float32)
+    return round_bf16(x) if dtype == "bf16" else x
+
+
+def similarity_inputs(rows, T, D, seed, dtype="fp32", changed=0.1):
+    """Current / cached representations for the selection test.
+
+    Most tokens move a little between steps, a `changed` fraction moves a lot
+    (the tokens decoded at the last step); token 1 duplicates token 0 (an exact
+    tie), token 2 is the zero vector when T > 2.
+    """
+    rng = np.random.Generator(np.random.PCG64(seed))
+    ref = rng.standard_normal((rows, T, D), dtype=np.float32)
+    cur = ref + np.float32(0.05) * rng.standard_normal((rows, T, D), dtype=np.float32)
+    big = rng.random((rows, T)) < changed
+    cur[big] = rng.standard_normal((int(big.sum()), D), dtype=np.float32)
+    if T > 1:
+        cur[:, 1], ref[:, 1] = cur[:, 0], ref[:, 0]
+    if T > 2:
+        cur[:, 2] = 0.0
+    if dtype == "bf16":
+        cur, ref = round_bf16(cur), round_bf16(ref)
+    return cur.astype(np.float32), ref.astype(np.float32)
+
+
+def distinct_rows(n, total, seed):
+    """n distinct row indices out of `total`, in random order (a scatter map)."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    return rng.permutation(total)[:n].astype(np.int32)

@@ -1,0 +1,181 @@
+"""Kernel-level parity: each CUDA kernel, called through the C ABI, against
+the CPU oracle on the same seeded inputs."""
+import numpy as np
+import pytest
+
+import oracle as O
+import synth
+from paper_2503_12450_gb300 import lazymar as lm
+from _gpu import DT, TOL, dev, dev_int, empty, host, max_rel, sync, torch_cuda
+
+pytestmark = pytest.mark.gpu
+
+
+# --------------------------------------------------------------------------
+# Selection (Eq. 8): indices bit-exact
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("rows,T,D,N,dtype", [
+    (2, 80, 256, 20, "fp32"),      # tiny
+    (64, 320, 768, 50, "bf16"),    # MAR-B
+    (16, 320, 1024, 32, "bf16"),   # MAR-L, 10 %
+    (8, 320, 1280, 50, "bf16"),    # MAR-H
+    (32, 1088, 1024, 272, "bf16"),  # high resolution, 25 %
+    (3, 320, 768, 0, "bf16"),
+    (3, 320, 768, 320, "bf16"),
+    (1, 1, 8, 1, "fp32"),
+    (5, 100, 16, 37, "bf16"),
+    (4, 513, 64, 129, "fp32"),     # T spans two scan chunks
+])
+def test_select_tokens_bit_exact(rows, T, D, N, dtype):
+    torch = torch_cuda()
+    cur, ref = synth.similarity_inputs(rows, T, D, seed=rows * 1000 + T, dtype=dtype)
+    g_cur, g_ref = dev(cur, dtype), dev(ref, dtype)
+    idx = torch.full((rows, max(N, 1)), -1, dtype=torch.int32, device="cuda")
+    lm.lazymar_select_tokens(DT[dtype], g_cur, g_ref, rows, T, D, N, idx)
+    sync()
+    got = idx.cpu().numpy()[:, :N]
+    for r in range(rows):
+        expect = O.select_compute(O.cosine_similarity(cur[r], ref[r]), N)
+        assert got[r].tolist() == expect.tolist(), "row %d" % r
+    # the reference now holds the current values, bit for bit
+    assert torch.equal(g_ref, g_cur)
+
+
+# --------------------------------------------------------------------------
+# Condition cache / guidance (Eq. 7 reading, Eq. 10)
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+@pytest.mark.parametrize("mode", [lm.LAZYMAR_CFG_GUIDE, lm.LAZYMAR_CFG_REFRESH, lm.LAZYMAR_CFG_REUSE])
+@pytest.mark.parametrize("n", [8 * 1000 + 3, 32 * 256 * 768])
+def test_cfg_combine(dtype, mode, n):
+    gamma = 3.0
+    c = synth.tensor((n,), 11, dtype=dtype)
+    u = synth.tensor((n,), 12, dtype=dtype)
+    d = synth.tensor((n,), 13, std=0.1, dtype=dtype)
+    gc, gu, gd = dev(c, dtype), dev(u, dtype), dev(d, dtype)
+    g, uo = empty((n,), dtype), empty((n,), dtype)
+    lm.lazymar_cfg_combine(DT[dtype], mode, gc, gu, gd, gamma, n, uo, g)
+    sync()
+    tol = 8e-3 if dtype == "bf16" else 1e-6
+    if mode == lm.LAZYMAR_CFG_REUSE:
+        u_ref = O.cond_cache_reuse(c, d)
+        assert max_rel(host(uo), u_ref) < tol
+    else:
+        u_ref = u
+    if mode == lm.LAZYMAR_CFG_REFRESH:
+        assert max_rel(host(gd), O.cond_cache_store(c, u)) < tol
+    assert max_rel(host(g), O.guidance(c, u_ref, gamma)) < tol
+
+
+# --------------------------------------------------------------------------
+# GEMMs (tcgen05 for bf16, CUDA cores for fp32) with every epilogue
+# --------------------------------------------------------------------------
+
+GEMM_SHAPES = [
+    (1, 384, 128), (40, 768, 256), (200, 2304, 768), (3200, 2304, 768), (3200, 768, 768),
+    (3200, 3072, 768), (3200, 768, 3072), (777, 1280, 1280), (384, 3840, 1280),
+]
+
+
+def _linear_case(dtype, epi, M, N, K, flags, seed):
+    torch = torch_cuda()
+    a = synth.tensor((M, K), seed, dtype=dtype)
+    w = synth.tensor((N, K), seed + 1, std=0.05, dtype=dtype)
+    b = synth.tensor((N,), seed + 2, std=0.1, dtype=dtype)
+    ga, gw, gb = dev(a, dtype), dev(w, dtype), dev(b, dtype)
+    ref = O.linear(a, w, b)
+    out_dtype_tol = 1e-2 if dtype == "bf16" else 1e-4
+    if epi in (lm.LAZYMAR_EPI_BIAS, lm.LAZYMAR_EPI_GELU):
+        out = empty((M, N), dtype)
+        lm.lazymar_linear(DT[dtype], epi, ga, gw, gb, M, N, K, out, N, flags=flags)
+        sync()
+        expect = ref if epi == lm.LAZYMAR_EPI_BIAS else O.gelu(ref)
+        assert max_rel(host(out), expect) < out_dtype_tol
+    elif epi == lm.LAZYMAR_EPI_RESIDUAL:
+        r0 = synth.tensor((M, N), seed + 3)
+        out = dev(r0, "fp32")
+        lm.lazymar_linear(DT[dtype], epi, ga, gw, gb, M, N, K, out, N, flags=flags)
+        sync()
+        assert max_rel(host(out), r0 + ref) < 1e-4
+    else:
+        D = N // 3
+        R = M + 17
+        row_map = synth.distinct_rows(M, R, seed + 4)
+        k0 = synth.tensor((R, D), seed + 5, dtype=dtype)
+        v0 = synth.tensor((R, D), seed + 6, dtype=dtype)
+        q, gk, gv = empty((M, D), dtype), dev(k0, dtype), dev(v0, dtype)
+        lm.lazymar_linear(DT[dtype], epi, ga, gw, gb, M, N, K, q, D, gk, gv, dev_int(row_map), flags=flags)
+        sync()
+        assert max_rel(host(q), ref[:, :D]) < out_dtype_tol
+        k, v = host(gk), host(gv)
+        assert max_rel(k[row_map], ref[:, D:2 * D]) < out_dtype_tol
+        assert max_rel(v[row_map], ref[:, 2 * D:]) < out_dtype_tol
+        keep = np.setdiff1d(np.arange(R), row_map)
+        assert np.array_equal(k[keep], k0[keep]) and np.array_equal(v[keep], v0[keep])
+
+
+@pytest.mark.parametrize("M,N,K", GEMM_SHAPES)
+@pytest.mark.parametrize("epi", [lm.LAZYMAR_EPI_BIAS, lm.LAZYMAR_EPI_GELU, lm.LAZYMAR_EPI_RESIDUAL,
+                                 lm.LAZYMAR_EPI_QKV])
+def test_linear_bf16_tcgen05(M, N, K, epi):
+    if epi == lm.LAZYMAR_EPI_QKV and (N % 3 or (N // 3) % 32):
+        pytest.skip("not a QKV shape")
+    for flags in ([1, 2] if N % 256 == 0 else [1]):
+        _linear_case("bf16", epi, M, N, K, flags, seed=M + N + K + epi)
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 12, 8), (40, 768, 256), (160, 1024, 256), (77, 256, 1024)])
+@pytest.mark.parametrize("epi", [lm.LAZYMAR_EPI_BIAS, lm.LAZYMAR_EPI_GELU, lm.LAZYMAR_EPI_RESIDUAL,
+                                 lm.LAZYMAR_EPI_QKV])
+def test_linear_fp32(M, N, K, epi):
+    if epi == lm.LAZYMAR_EPI_QKV and (N % 3 or (N // 3) % 4):
+        pytest.skip("not a QKV shape")
+    _linear_case("fp32", epi, M, N, K, 0, seed=M + N + K + epi)
+
+
+# --------------------------------------------------------------------------
+# Attention (Eq. 3 with a query subset)
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("rows,n_q,T,heads,dh,dtype", [
+    (2, 50, 320, 12, 64, "bf16"),    # MAR-B cached layer
+    (2, 320, 320, 4, 64, "bf16"),    # full layer
+    (1, 272, 1088, 2, 64, "bf16"),   # high resolution cached layer
+    (3, 50, 320, 4, 80, "bf16"),     # MAR-H head width
+    (2, 65, 130, 2, 80, "bf16"),     # ragged queries and keys
+    (1, 1, 1, 1, 64, "bf16"),
+    (2, 20, 80, 4, 64, "fp32"),      # tiny
+    (1, 3, 5, 2, 32, "fp32"),
+])
+def test_attention(rows, n_q, T, heads, dh, dtype):
+    D = heads * dh
+    q = synth.tensor((rows, n_q, D), 21, dtype=dtype)
+    k = synth.tensor((rows, T, D), 22, dtype=dtype)
+    v = synth.tensor((rows, T, D), 23, dtype=dtype)
+    o = empty((rows, n_q, D), dtype)
+    lm.lazymar_attention(DT[dtype], dev(q, dtype), dev(k, dtype), dev(v, dtype), o, rows, n_q, T, heads, dh)
+    sync()
+    ref = np.stack([O.attention(q[r], k[r], v[r], heads) for r in range(rows)])
+    assert max_rel(host(o), ref) < (1e-2 if dtype == "bf16" else 1e-5)
+
+
+# --------------------------------------------------------------------------
+# LayerNorm (gathering rows)
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("M,D,gather,dtype", [(100, 768, False, "bf16"), (50, 1280, True, "bf16"),
+                                              (80, 256, True, "fp32"), (3, 1024, False, "fp32")])
+def test_layernorm(M, D, gather, dtype):
+    R = M + 30
+    x = synth.tensor((R, D), 31, std=2.0, mean=0.5)
+    g = synth.tensor((D,), 32, std=0.1, mean=1.0, dtype=dtype)
+    b = synth.tensor((D,), 33, std=0.1, dtype=dtype)
+    rm = synth.distinct_rows(M, R, 34) if gather else None
+    y = empty((M, D), dtype)
+    lm.lazymar_layernorm(DT[dtype], dev(x), None if rm is None else dev_int(rm), dev(g, dtype), dev(b, dtype), y,
+                         M, D, 1e-6)
+    sync()
+    src = x[rm] if gather else x[:M]
+    assert max_rel(host(y), O.layer_norm(src, g, b, 1e-6)) < (1e-2 if dtype == "bf16" else 1e-5)
