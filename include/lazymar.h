@@ -222,6 +222,16 @@ lazymar_status lazymar_layernorm(int dtype, const float *x, const int32_t *row_m
  * condition cache, or -1 for invalid arguments. */
 int lazymar_plan_step(int k, int k0, int tau, int tau_cfg, int use_cond_cache);
 
+/* Step execution. Each step first copies its inputs (latents, mask, labels,
+ * idx_in) into handle-owned buffers on `stream`, so the device work reads
+ * fixed addresses. That work (embedding through the final LayerNorm) runs
+ * eagerly the first time a (step kind, B, N, cond reuse, idx_in given)
+ * combination is seen, is captured into a CUDA graph the second time and
+ * replayed from then on; the CFG combine and the output copies are launched
+ * after it, so gamma may change from call to call. enable = 0 runs every step
+ * eagerly. Graphs are never used while profiling is on. */
+lazymar_status lazymar_set_graphs(lazymar_handle *h, int enable);
+
 /* Waits for `stream`, then reports (and clears) errors the handle's kernels
  * latched on the device: TIMEOUT, DEVICE, or CUDA for an asynchronous fault. */
 lazymar_status lazymar_sync(lazymar_handle *h, void *stream);

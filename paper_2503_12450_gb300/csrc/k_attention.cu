@@ -188,8 +188,12 @@ __global__ void __launch_bounds__(128) attention_bf16_kernel(const __grid_consta
         mma_bf16_16816(oacc[nb + 1], pa, b2, b3);
       }
     }
-    __syncthreads();  // every warp is done with this stage
+    // Every warp has consumed its ldmatrix reads of this stage (the mma that
+    // uses them precedes the barrier); the proxy fence then orders those
+    // generic-proxy reads before the async-proxy TMA that refills the stage.
+    __syncthreads();
     if (tid == 0 && j + 2 < nkt) {
+      fence_proxy_async_smem();
       const int jn = j + 2;
       mbar_arrive_expect_tx(&bars[1 + st], kv_bytes);
       tma_load_2d(&tmK, &bars[1 + st], sK + st * at::TILE64, col, kv0 + jn * at::KT);

@@ -190,29 +190,56 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
     __syncwarp();
   } else {
     // ---------------- epilogue warps ----------------
+    // The fp32 residual of a chunk does not depend on the accumulator, so the
+    // first chunk's residual is loaded before waiting for the accumulator and
+    // each later chunk's while the previous one is processed: the global-load
+    // latency overlaps the main loop instead of stalling the epilogue.
     const int ew = warp - 2;        // 0..7
     const int quarter = warp & 3;   // tensor-memory lanes this warp may read
     const int half = ew >> 2;       // which half of the tile's columns
     constexpr int CHUNKS = BN / 64; // 32-column chunks per half
+    const bool resid = epi.mode == LAZYMAR_EPI_RESIDUAL;
+    float* const res_base = static_cast<float*>(epi.out);
     int it = 0;
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++it) {
       const int buf = it & 1;
       const uint32_t use = (uint32_t)(it >> 1) & 1u;
+      const int m0 = (tile % num_m) * tc::BM, n0 = (tile / num_m) * BN;
+      const int row = m0 + quarter * 32 + lane;
+      const bool row_ok = row < M;
+      const int c0 = half * CHUNKS;
+      float nxt[32];
+      if (resid && row_ok) Vec<float, 32>::load(res_base + (size_t)row * epi.ldo + n0 + c0 * 32, nxt);
       const bool ok = mbar_wait(&acc_full[buf], use, abort_flag, err);
       if (__any_sync(0xffffffffu, !ok)) break;
       tc_fence_after();
-      const int m0 = (tile % num_m) * tc::BM, n0 = (tile / num_m) * BN;
-      const int row = m0 + quarter * 32 + lane;
 #pragma unroll 1
-      for (int c = half * CHUNKS; c < (half + 1) * CHUNKS; ++c) {
+      for (int c = c0; c < c0 + CHUNKS; ++c) {
+        const int col = n0 + c * 32;
+        float res[32];
+        if (resid) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) res[i] = nxt[i];
+          if (row_ok && c + 1 < c0 + CHUNKS) Vec<float, 32>::load(res_base + (size_t)row * epi.ldo + col + 32, nxt);
+        }
         uint32_t r[32];
         tmem_ld32(tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN + c * 32), r);
+        float bv[32];
+        if (epi.bias) Vec<bf16, 32>::load(static_cast<const bf16*>(epi.bias) + col, bv);
         tmem_wait_ld();
-        if (row < M) {
+        if (row_ok) {
           float v[32];
 #pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-          epilogue_apply<bf16, 32>(epi, row, n0 + c * 32, v);
+          for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]) + (epi.bias ? bv[i] : 0.f);
+          if (resid) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] += res[i];
+            Vec<float, 32>::store(res_base + (size_t)row * epi.ldo + col, v);
+          } else {
+            GemmEpi e2 = epi;
+            e2.bias = nullptr;
+            epilogue_apply<bf16, 32>(e2, row, col, v);
+          }
         }
       }
       tc_fence_before();
@@ -361,7 +388,7 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
     const long mt = (M + tc::BM - 1) / tc::BM;
     const long w128 = (mt * (N / 128) + c.num_sms - 1) / c.num_sms * 128;
     const long w256 = (mt * (N / 256) + c.num_sms - 1) / c.num_sms * 256;
-    if (w256 <= w128) bn = 256;
+    if (w256 * 100 <= w128 * 115) bn = 256;  // BN = 256 has the more efficient main loop
   }
   return bn == 256 ? launch_tc<256>(c, A, W, M, N, K, epi) : launch_tc<128>(c, A, W, M, N, K, epi);
 }

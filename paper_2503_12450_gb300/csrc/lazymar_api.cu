@@ -6,6 +6,8 @@
 #include <mutex>
 #include <string>
 #include <vector>
+#include <map>
+#include <tuple>
 
 #include "lazymar_internal.cuh"
 
@@ -121,6 +123,22 @@ struct lazymar_handle {
   };
   std::vector<Ev> evs;
   size_t ev_used = 0;
+  // CUDA graphs of step bodies, keyed by (kind, batch, N, cond reuse, caller indices)
+  struct GraphKey {
+    int kind, B, N, reuse, idx;
+    bool operator<(const GraphKey& o) const {
+      return std::tie(kind, B, N, reuse, idx) < std::tie(o.kind, o.B, o.N, o.reuse, o.idx);
+    }
+  };
+  struct GraphEntry {
+    cudaGraphExec_t exec = nullptr;
+    int eager_runs = 0;
+    lazymar_stats delta{};
+  };
+  std::map<GraphKey, GraphEntry> graphs;
+  bool use_graphs = true;
+  cudaStream_t gstream = nullptr;  // capture / replay stream
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
 };
 
 namespace {
@@ -316,6 +334,10 @@ extern "C" lazymar_status lazymar_create(const lazymar_config* cfg, const lazyma
 
   e = cudaMemset(h->arena, 0, h->arena_bytes);
   if (e != cudaSuccess) return destroy(cuda_fail(e, "cudaMemset"));
+  if ((e = cudaStreamCreateWithFlags(&h->gstream, cudaStreamNonBlocking)) != cudaSuccess ||
+      (e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming)) != cudaSuccess ||
+      (e = cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming)) != cudaSuccess)
+    return destroy(cuda_fail(e, "stream/event creation"));
   lazymar_status st;
   const int dt = cfg->dtype;
   if ((st = upload(h->pos, w->pos_emb, T * D, dt)) || (st = upload(h->cls, w->class_emb, (size_t)cfg->n_classes * D, dt)) ||
@@ -341,6 +363,11 @@ extern "C" lazymar_status lazymar_create(const lazymar_config* cfg, const lazyma
 extern "C" void lazymar_destroy(lazymar_handle* h) {
   if (!h) return;
   DeviceGuard g(h->dev);
+  for (auto& kv : h->graphs)
+    if (kv.second.exec) cudaGraphExecDestroy(kv.second.exec);
+  if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+  if (h->ev_join) cudaEventDestroy(h->ev_join);
+  if (h->gstream) cudaStreamDestroy(h->gstream);
   for (auto& e : h->evs) {
     cudaEventDestroy(e.a);
     cudaEventDestroy(e.b);
@@ -354,31 +381,15 @@ extern "C" void lazymar_destroy(lazymar_handle* h) {
 // ---------------------------------------------------------------------------
 namespace {
 
-struct StepInputs {
-  const float* lat;
-  const uint8_t* mask;
-  const int* labels;
-};
-
-lazymar_status stage_inputs(lazymar_handle* h, const lazymar_step_in* in, cudaStream_t st, StepInputs* io) {
+// Step inputs always go through the handle's staging buffers, so the device
+// work of a step reads fixed addresses and can be replayed from a CUDA graph.
+lazymar_status stage_inputs(lazymar_handle* h, const lazymar_step_in* in, cudaStream_t st) {
   const int B = in->batch;
   const size_t nl = (size_t)B * h->cfg.n_img * h->cfg.token_dim;
   const size_t nm = (size_t)B * h->cfg.n_img;
-  io->lat = in->latents;
-  io->mask = in->mask;
-  io->labels = in->labels;
-  if (!is_device_ptr(in->latents)) {
-    LM_CUDA(cudaMemcpyAsync(h->st_lat, in->latents, nl * 4, cudaMemcpyHostToDevice, st));
-    io->lat = h->st_lat;
-  }
-  if (!is_device_ptr(in->mask)) {
-    LM_CUDA(cudaMemcpyAsync(h->st_mask, in->mask, nm, cudaMemcpyHostToDevice, st));
-    io->mask = h->st_mask;
-  }
-  if (!is_device_ptr(in->labels)) {
-    LM_CUDA(cudaMemcpyAsync(h->st_labels, in->labels, (size_t)B * 4, cudaMemcpyHostToDevice, st));
-    io->labels = h->st_labels;
-  }
+  LM_CUDA(cudaMemcpyAsync(h->st_lat, in->latents, nl * 4, cudaMemcpyDefault, st));
+  LM_CUDA(cudaMemcpyAsync(h->st_mask, in->mask, nm, cudaMemcpyDefault, st));
+  LM_CUDA(cudaMemcpyAsync(h->st_labels, in->labels, (size_t)B * 4, cudaMemcpyDefault, st));
   return LAZYMAR_OK;
 }
 
@@ -455,10 +466,10 @@ lazymar_status layer_cached(lazymar_handle* h, const Ctx& c, int l, int rows, in
   return LAZYMAR_OK;
 }
 
-lazymar_status embed(lazymar_handle* h, const Ctx& c, const StepInputs& io, int rows, int B) {
+lazymar_status embed(lazymar_handle* h, const Ctx& c, int rows, int B) {
   const double bytes = (double)rows * h->T * h->D * (4.0 + h->es);
   return launch(h, LAZYMAR_K_EMBED, 0, bytes, c.stream, "embed", [&] {
-    return launch_embed(c, h->cfg.dtype, io.lat, io.mask, io.labels, h->pos, h->cls, h->memb, h->ew, h->eb, h->H, rows,
+    return launch_embed(c, h->cfg.dtype, h->st_lat, h->st_mask, h->st_labels, h->pos, h->cls, h->memb, h->ew, h->eb, h->H, rows,
                         B, h->T, h->cfg.n_buffer, h->cfg.n_img, h->D, h->cfg.token_dim, h->cfg.n_classes);
   });
 }
@@ -485,6 +496,105 @@ lazymar_status cfg(lazymar_handle* h, const Ctx& c, int mode, int B, float gamma
 // pointers through the staging buffer `st` and a copy at the end.
 void* out_target(void* user, void* st) { return user == nullptr ? nullptr : (is_device_ptr(user) ? user : st); }
 
+// Device work of a full step up to the output cache (everything but the CFG
+// combine, which takes gamma and stays outside any graph).
+lazymar_status full_body(lazymar_handle* h, const Ctx& c, int B) {
+  const int rows = 2 * B, s = h->s;
+  LM_TRY(embed(h, c, rows, B));
+  for (int l = 0; l < h->L; ++l) {
+    const bool value_ref = l == s - 1 && h->cfg.criterion == LAZYMAR_CRITERION_VALUE;
+    void* kdst = l >= s ? h->Kc[l] : h->Ks;
+    void* vdst = l >= s ? h->Vc[l] : (value_ref ? h->ref : h->Vs);
+    LM_TRY(layer_full(h, c, l, rows, kdst, vdst));
+    if (l == s - 1 && h->cfg.criterion == LAZYMAR_CRITERION_FEATURE) {
+      const size_t n = (size_t)rows * h->T * h->D;
+      LM_TRY(launch(h, LAZYMAR_K_OTHER, 0, n * (4.0 + h->es), c.stream, "cast",
+                    [&] { return launch_cast(c, h->cfg.dtype, h->H, h->ref, n); }));
+    }
+  }
+  return final_ln(h, c, h->H, nullptr, rows * h->T);
+}
+
+// Device work of a cached step up to the output cache.
+lazymar_status cached_body(lazymar_handle* h, const Ctx& c, int rows, int N, bool has_idx) {
+  const int s = h->s, T = h->T, D = h->D;
+  LM_TRY(embed(h, c, rows, h->last_batch));
+  for (int l = 0; l < s; ++l) LM_TRY(layer_full(h, c, l, rows, h->Ks, h->Vs));
+  // Eq. 8: similarity of block s-1's representation with the reference, then
+  // the reference takes this step's values.
+  const void* cur = h->Vs;
+  if (h->cfg.criterion == LAZYMAR_CRITERION_FEATURE) {
+    const size_t n = (size_t)rows * T * D;
+    LM_TRY(launch(h, LAZYMAR_K_OTHER, 0, n * (4.0 + h->es), c.stream, "cast",
+                  [&] { return launch_cast(c, h->cfg.dtype, h->H, h->Fs, n); }));
+    cur = h->Fs;
+  }
+  LM_TRY(launch(h, LAZYMAR_K_SELECT, 0, 3.0 * rows * T * D * h->es + 8.0 * rows * T, c.stream, "similarity",
+                [&] { return launch_similarity(c, h->cfg.dtype, cur, h->ref, h->S, rows, T, D, true); }));
+  if (has_idx) {
+    LM_TRY(launch(h, LAZYMAR_K_SELECT, 0, 12.0 * rows * N, c.stream, "index check",
+                  [&] { return launch_idx_check(c, h->st_idx_in, rows, T, N, h->idx, h->row_map); }));
+  } else if (N > 0) {
+    LM_TRY(launch(h, LAZYMAR_K_SELECT, 0, 8.0 * rows * T + 8.0 * rows * N, c.stream, "topk",
+                  [&] { return launch_topk(c, h->S, rows, T, N, h->idx, h->row_map); }));
+  }
+  if (N > 0) {
+    for (int l = s; l < h->L; ++l) LM_TRY(layer_cached(h, c, l, rows, N, l == s));
+    LM_TRY(final_ln(h, c, h->Hc, h->row_map, rows * N));
+  }
+  return LAZYMAR_OK;
+}
+
+void add_stats(lazymar_stats& a, const lazymar_stats& d, double sign) {
+  for (int i = 0; i < LAZYMAR_K_COUNT; ++i) {
+    a.k[i].launches += (long long)sign * d.k[i].launches;
+    a.k[i].flops += sign * d.k[i].flops;
+    a.k[i].bytes += sign * d.k[i].bytes;
+  }
+}
+
+// Runs a step body: eagerly on the caller's stream on its first use (and
+// always while profiling or with graphs disabled); from then on as a CUDA
+// graph, captured on the second use and replayed afterwards. Capture and
+// replay run on the handle's own stream, joined to the caller's stream by
+// events (the legacy default stream cannot be captured).
+template <class F>
+lazymar_status run_body(lazymar_handle* h, cudaStream_t st, const lazymar_handle::GraphKey& key, F&& body) {
+  if (h->profiling || !h->use_graphs) return body(Ctx{st, h->err, h->num_sms});
+  lazymar_handle::GraphEntry& ge = h->graphs[key];
+  if (!ge.exec && ge.eager_runs++ == 0) return body(Ctx{st, h->err, h->num_sms});
+  cudaStream_t gs = h->gstream;
+  LM_CUDA(cudaEventRecord(h->ev_fork, st));
+  LM_CUDA(cudaStreamWaitEvent(gs, h->ev_fork, 0));
+  if (!ge.exec) {
+    const lazymar_stats before = h->stats;
+    LM_CUDA(cudaStreamBeginCapture(gs, cudaStreamCaptureModeThreadLocal));
+    const lazymar_status s = body(Ctx{gs, h->err, h->num_sms});
+    cudaGraph_t g = nullptr;
+    const cudaError_t e = cudaStreamEndCapture(gs, &g);
+    if (s != LAZYMAR_OK || e != cudaSuccess) {
+      if (g) cudaGraphDestroy(g);
+      h->stats = before;
+      return s != LAZYMAR_OK ? s : cuda_fail(e, "cudaStreamEndCapture");
+    }
+    const cudaError_t ei = cudaGraphInstantiate(&ge.exec, g, 0);
+    cudaGraphDestroy(g);
+    if (ei != cudaSuccess) {
+      ge.exec = nullptr;
+      h->stats = before;
+      return cuda_fail(ei, "cudaGraphInstantiate");
+    }
+    ge.delta = h->stats;
+    add_stats(ge.delta, before, -1.0);
+    h->stats = before;
+  }
+  LM_CUDA(cudaGraphLaunch(ge.exec, gs));
+  LM_CUDA(cudaEventRecord(h->ev_join, gs));
+  LM_CUDA(cudaStreamWaitEvent(st, h->ev_join, 0));
+  add_stats(h->stats, ge.delta, 1.0);
+  return LAZYMAR_OK;
+}
+
 }  // namespace
 
 extern "C" lazymar_status lazymar_full_step(lazymar_handle* h, const lazymar_step_in* in, float gamma, void* z_out,
@@ -493,25 +603,12 @@ extern "C" lazymar_status lazymar_full_step(lazymar_handle* h, const lazymar_ste
   DeviceGuard dg(h->dev);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const Ctx c{st, h->err, h->num_sms};
-  const int B = in->batch, rows = 2 * B, s = h->s;
-  StepInputs io;
-  LM_TRY(stage_inputs(h, in, st, &io));
-  LM_TRY(embed(h, c, io, rows, B));
-  for (int l = 0; l < h->L; ++l) {
-    const bool value_ref = l == s - 1 && h->cfg.criterion == LAZYMAR_CRITERION_VALUE;
-    void* kdst = l >= s ? h->Kc[l] : h->Ks;
-    void* vdst = l >= s ? h->Vc[l] : (value_ref ? h->ref : h->Vs);
-    LM_TRY(layer_full(h, c, l, rows, kdst, vdst));
-    if (l == s - 1 && h->cfg.criterion == LAZYMAR_CRITERION_FEATURE) {
-      const size_t n = (size_t)rows * h->T * h->D;
-      LM_TRY(launch(h, LAZYMAR_K_OTHER, 0, n * (4.0 + h->es), st, "cast",
-                    [&] { return launch_cast(c, h->cfg.dtype, h->H, h->ref, n); }));
-    }
-  }
-  LM_TRY(final_ln(h, c, h->H, nullptr, rows * h->T));
+  const int B = in->batch;
+  LM_TRY(stage_inputs(h, in, st));
+  LM_TRY(run_body(h, st, lazymar_handle::GraphKey{0, B, 0, 0, 0}, [&](const Ctx& cc) { return full_body(h, cc, B); }));
   void* g_dst = out_target(guided_out, h->st_g);
   LM_TRY(cfg(h, c, LAZYMAR_CFG_REFRESH, B, gamma, nullptr, g_dst));
-  const size_t zbytes = (size_t)rows * h->cfg.n_img * h->D * h->es;
+  const size_t zbytes = (size_t)2 * B * h->cfg.n_img * h->D * h->es;
   if (z_out) LM_CUDA(cudaMemcpyAsync(z_out, h->zc, zbytes, cudaMemcpyDefault, st));
   if (guided_out && g_dst != guided_out)
     LM_CUDA(cudaMemcpyAsync(guided_out, g_dst, zbytes / 2, cudaMemcpyDeviceToHost, st));
@@ -530,39 +627,12 @@ extern "C" lazymar_status lazymar_cached_step(lazymar_handle* h, const lazymar_s
   DeviceGuard dg(h->dev);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const Ctx c{st, h->err, h->num_sms};
-  const int B = in->batch, rows = use_cond_cache ? B : 2 * B, s = h->s, N = n_compute, T = h->T, D = h->D;
-  StepInputs io;
-  LM_TRY(stage_inputs(h, in, st, &io));
-  LM_TRY(embed(h, c, io, rows, B));
-  for (int l = 0; l < s; ++l) LM_TRY(layer_full(h, c, l, rows, h->Ks, h->Vs));
-
-  // Eq. 8: similarity of block s-1's representation with the reference, then
-  // the reference takes this step's values.
-  const void* cur = h->Vs;
-  if (h->cfg.criterion == LAZYMAR_CRITERION_FEATURE) {
-    const size_t n = (size_t)rows * T * D;
-    LM_TRY(launch(h, LAZYMAR_K_OTHER, 0, n * (4.0 + h->es), st, "cast",
-                  [&] { return launch_cast(c, h->cfg.dtype, h->H, h->Fs, n); }));
-    cur = h->Fs;
-  }
-  LM_TRY(launch(h, LAZYMAR_K_SELECT, 0, 3.0 * rows * T * D * h->es + 8.0 * rows * T, st, "similarity",
-                [&] { return launch_similarity(c, h->cfg.dtype, cur, h->ref, h->S, rows, T, D, true); }));
-  if (idx_in) {
-    const int* src = idx_in;
-    if (!is_device_ptr(idx_in)) {
-      LM_CUDA(cudaMemcpyAsync(h->st_idx_in, idx_in, (size_t)rows * N * 4, cudaMemcpyHostToDevice, st));
-      src = h->st_idx_in;
-    }
-    LM_TRY(launch(h, LAZYMAR_K_SELECT, 0, 12.0 * rows * N, st, "index check",
-                  [&] { return launch_idx_check(c, src, rows, T, N, h->idx, h->row_map); }));
-  } else if (N > 0) {
-    LM_TRY(launch(h, LAZYMAR_K_SELECT, 0, 8.0 * rows * T + 8.0 * rows * N, st, "topk",
-                  [&] { return launch_topk(c, h->S, rows, T, N, h->idx, h->row_map); }));
-  }
-  if (N > 0) {
-    for (int l = s; l < h->L; ++l) LM_TRY(layer_cached(h, c, l, rows, N, l == s));
-    LM_TRY(final_ln(h, c, h->Hc, h->row_map, rows * N));
-  }
+  const int B = in->batch, rows = use_cond_cache ? B : 2 * B, N = n_compute, D = h->D;
+  LM_TRY(stage_inputs(h, in, st));
+  const bool has_idx = idx_in != nullptr && N > 0;
+  if (has_idx) LM_CUDA(cudaMemcpyAsync(h->st_idx_in, idx_in, (size_t)rows * N * 4, cudaMemcpyDefault, st));
+  LM_TRY(run_body(h, st, lazymar_handle::GraphKey{1, B, N, use_cond_cache ? 1 : 0, has_idx ? 1 : 0},
+                  [&](const Ctx& cc) { return cached_body(h, cc, rows, N, has_idx); }));
 
   const size_t n_el = (size_t)B * h->cfg.n_img * D;
   void* z_dst = out_target(z_out, h->st_z);
@@ -579,6 +649,12 @@ extern "C" lazymar_status lazymar_cached_step(lazymar_handle* h, const lazymar_s
   if (guided_out && g_dst != guided_out)
     LM_CUDA(cudaMemcpyAsync(guided_out, g_dst, n_el * h->es, cudaMemcpyDeviceToHost, st));
   if (idx_out && N > 0) LM_CUDA(cudaMemcpyAsync(idx_out, h->idx, (size_t)rows * N * 4, cudaMemcpyDefault, st));
+  return LAZYMAR_OK;
+}
+
+extern "C" lazymar_status lazymar_set_graphs(lazymar_handle* h, int enable) {
+  if (!h) return fail(LAZYMAR_ERR_INVALID_ARG, "NULL handle");
+  h->use_graphs = enable != 0;
   return LAZYMAR_OK;
 }
 

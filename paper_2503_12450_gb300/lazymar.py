@@ -86,6 +86,7 @@ def lib():
         "lazymar_sync": (st, [vp, vp]),
         "lazymar_device_check": (st, [vp]),
         "lazymar_set_profiling": (st, [vp, i]),
+        "lazymar_set_graphs": (st, [vp, i]),
         "lazymar_get_stats": (st, [vp, ctypes.POINTER(lazymar_stats)]),
         "lazymar_reset_stats": (st, [vp]),
         "lazymar_status_string": (ctypes.c_char_p, [i]),
@@ -234,6 +235,10 @@ def lazymar_device_check(stream=None):
 
 def lazymar_set_profiling(h, enable):
     _check(lib().lazymar_set_profiling(h.ptr, int(bool(enable))))
+
+
+def lazymar_set_graphs(h, enable):
+    _check(lib().lazymar_set_graphs(h.ptr, int(bool(enable))))
 
 
 def lazymar_get_stats(h):
