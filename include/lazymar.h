@@ -171,6 +171,25 @@ lazymar_status lazymar_cached_step(lazymar_handle *h, const lazymar_step_in *in,
 lazymar_status lazymar_select_tokens(int dtype, const void *v_cur, void *v_cache, int rows, int T,
                                      int D, int n_compute, int32_t *idx_out, void *stream);
 
+/* lazymar_select_tokens without any device allocation. The paper has no
+ * counterpart: this entry point exists for callers that may not allocate
+ * device memory once running (a serving loop that fixes its memory budget at
+ * start-up, a plug-in whose host framework owns the device allocator). Same
+ * arguments, semantics and results as lazymar_select_tokens; device pointers
+ * only. The similarity scratch is a fixed array inside the library, holding
+ * LAZYMAR_SELECT_NOALLOC_MAX_TOKENS doubles (2 MiB) on every device that loads
+ * it, until the process exits; rows * T above that limit returns
+ * LAZYMAR_ERR_INVALID_ARG. The first call on a device looks up the array's
+ * device address (make that first call before any stream capture). All calls
+ * share the one array and leave their similarities in it: calls whose work
+ * can overlap on the GPU (different streams, or different host threads) race
+ * and must be serialised by the caller. No cudaMalloc, cudaFree or other
+ * allocating call is made. */
+#define LAZYMAR_SELECT_NOALLOC_MAX_TOKENS 262144
+lazymar_status lazymar_select_tokens_noalloc(int dtype, const void *v_cur, void *v_cache, int rows,
+                                             int T, int D, int n_compute, int32_t *idx_out,
+                                             void *stream);
+
 /* Classifier-free guidance with the condition cache (Eq. 7 read as
  * u + gamma (c - u), Eq. 10), elementwise over n elements (device pointers):
  *   mode 0 GUIDE:   guided = u + gamma (c - u)

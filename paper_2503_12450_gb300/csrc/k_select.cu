@@ -16,6 +16,7 @@
 // block-wide ballot/prefix scan writes them in ascending index order together
 // with the gather/scatter row map r*T + t.
 #include <cfloat>
+#include <mutex>
 
 #include "lazymar_internal.cuh"
 
@@ -158,4 +159,79 @@ cudaError_t launch_idx_check(const Ctx& c, const int* in, int rows, int T, int N
   return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------------------
+// Selection without device allocation
+// ---------------------------------------------------------------------------
+// Some callers may not allocate device memory once they are running: a
+// serving loop that reserves its whole memory budget at start-up and must not
+// grow it, or a plug-in whose host framework owns the device allocator and
+// forbids direct cudaMalloc. lazymar_select_tokens_noalloc serves them: its
+// similarity scratch is this fixed, module-level array, which every GPU that
+// loads the library holds until the process exits (8 bytes per token,
+// 2 MiB in total).
+static __device__ __align__(256) double g_select_scratch[LAZYMAR_SELECT_NOALLOC_MAX_TOKENS];
+
+constexpr int kMaxDevices = 64;
+
+// On the host, the name g_select_scratch denotes a host-side stand-in, not
+// device memory: handing it to a kernel would fault or, where the GPU can
+// reach host memory, silently use the wrong memory. The device address is
+// looked up once per device, with that device current, and reused.
+static cudaError_t select_scratch(int dev, double** out) {
+  static std::mutex mu;
+  static double* addr[kMaxDevices] = {};
+  std::lock_guard<std::mutex> lock(mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_select_scratch);
+    if (e != cudaSuccess) return e;
+    addr[dev] = static_cast<double*>(p);
+  }
+  *out = addr[dev];
+  return cudaSuccess;
+}
+
+static bool noalloc_device_ptr(const void* p) {
+  cudaPointerAttributes a;
+  if (!p || cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
 }  // namespace lm
+
+extern "C" lazymar_status lazymar_select_tokens_noalloc(int dtype, const void* v_cur, void* v_cache, int rows, int T,
+                                                        int D, int n_compute, int32_t* idx_out, void* stream) {
+  using namespace lm;
+  if (dtype != LAZYMAR_F32 && dtype != LAZYMAR_BF16) return report_error(LAZYMAR_ERR_INVALID_ARG, "dtype");
+  if (rows < 0 || T < 1 || T > 16384 || D < 8 || D % 8 != 0 || n_compute < 0 || n_compute > T)
+    return report_error(LAZYMAR_ERR_INVALID_ARG,
+                        "rows >= 0, 1 <= T <= 16384, D % 8 == 0, 0 <= n_compute <= T required");
+  if ((long long)rows * T > LAZYMAR_SELECT_NOALLOC_MAX_TOKENS)
+    return report_error(LAZYMAR_ERR_INVALID_ARG,
+                        "rows * T exceeds LAZYMAR_SELECT_NOALLOC_MAX_TOKENS (262144), the size of the fixed "
+                        "scratch; use lazymar_select_tokens");
+  if (rows == 0) return LAZYMAR_OK;
+  if (!noalloc_device_ptr(v_cur) || !noalloc_device_ptr(v_cache) || (n_compute > 0 && !noalloc_device_ptr(idx_out)))
+    return report_error(LAZYMAR_ERR_INVALID_ARG, "v_cur, v_cache and idx_out must be device pointers");
+  if ((reinterpret_cast<uintptr_t>(v_cur) | reinterpret_cast<uintptr_t>(v_cache)) & 15u)
+    return report_error(LAZYMAR_ERR_INVALID_ARG, "16-byte alignment required");
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+    return report_error(LAZYMAR_ERR_CUDA, "cudaGetDevice failed or device index out of range");
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return report_error(LAZYMAR_ERR_CUDA, "cudaDeviceGetAttribute failed");
+  double* S = nullptr;
+  if (select_scratch(dev, &S) != cudaSuccess)
+    return report_error(LAZYMAR_ERR_CUDA, "cudaGetSymbolAddress of the selection scratch failed");
+  // Every S entry the top-N reads is written by the similarity pass of the
+  // same call first, so the scratch needs no clearing between calls.
+  const Ctx c{static_cast<cudaStream_t>(stream), nullptr, sms};
+  cudaError_t e = launch_similarity(c, dtype, v_cur, v_cache, S, rows, T, D, true);
+  if (e == cudaSuccess) e = launch_topk(c, S, rows, T, n_compute, idx_out, nullptr);
+  if (e != cudaSuccess) return report_error(LAZYMAR_ERR_CUDA, cudaGetErrorString(e));
+  return LAZYMAR_OK;
+}
+

@@ -26,6 +26,10 @@ static lazymar_status fail(lazymar_status s, const std::string& msg) {
   g_last_error = msg;
   return s;
 }
+namespace lm {
+lazymar_status report_error(lazymar_status s, const char* msg) { return fail(s, msg); }
+}  // namespace lm
+
 static lazymar_status cuda_fail(cudaError_t e, const char* what) {
   return fail(LAZYMAR_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
 }

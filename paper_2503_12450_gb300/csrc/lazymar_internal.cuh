@@ -299,4 +299,8 @@ cudaError_t launch_idx_check(const Ctx& c, const int* idx_in, int rows, int T, i
 cudaError_t launch_cfg(const Ctx& c, int dtype, int mode, const void* zc, const void* zu, void* delta,
                        float gamma, size_t n, void* zu_out, void* g_out);
 
+// Records `msg` as the calling thread's last error (lazymar_last_error) and
+// returns `s`.
+lazymar_status report_error(lazymar_status s, const char* msg);
+
 }  // namespace lm

@@ -78,6 +78,7 @@ def lib():
         "lazymar_full_step": (st, [vp, ctypes.POINTER(lazymar_step_in), f, vp, vp, vp]),
         "lazymar_cached_step": (st, [vp, ctypes.POINTER(lazymar_step_in), i, i, f, vp, vp, vp, vp, vp]),
         "lazymar_select_tokens": (st, [i, vp, vp, i, i, i, i, vp, vp]),
+        "lazymar_select_tokens_noalloc": (st, [i, vp, vp, i, i, i, i, vp, vp]),
         "lazymar_cfg_combine": (st, [i, i, vp, vp, vp, f, sz, vp, vp, vp]),
         "lazymar_linear": (st, [i, i, vp, vp, vp, i, i, i, vp, i, vp, vp, vp, i, vp]),
         "lazymar_attention": (st, [i, vp, vp, vp, vp, i, i, i, i, i, vp]),
@@ -192,6 +193,11 @@ def lazymar_cached_step(h, latents, mask, labels, batch, n_compute, use_cond_cac
 def lazymar_select_tokens(dtype, v_cur, v_cache, rows, T, D, n_compute, idx_out, stream=None):
     _check(lib().lazymar_select_tokens(int(dtype), _ptr(v_cur), _ptr(v_cache), int(rows), int(T), int(D),
                                        int(n_compute), _ptr(idx_out), _stream(stream)))
+
+
+def lazymar_select_tokens_noalloc(dtype, v_cur, v_cache, rows, T, D, n_compute, idx_out, stream=None):
+    _check(lib().lazymar_select_tokens_noalloc(int(dtype), _ptr(v_cur), _ptr(v_cache), int(rows), int(T), int(D),
+                                               int(n_compute), _ptr(idx_out), _stream(stream)))
 
 
 def lazymar_cfg_combine(dtype, mode, z_cond, z_uncond, delta, gamma, n, z_uncond_out=None, guided_out=None,
