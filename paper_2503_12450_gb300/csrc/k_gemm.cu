@@ -388,7 +388,11 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
     const long mt = (M + tc::BM - 1) / tc::BM;
     const long w128 = (mt * (N / 128) + c.num_sms - 1) / c.num_sms * 128;
     const long w256 = (mt * (N / 256) + c.num_sms - 1) / c.num_sms * 256;
-    if (w256 * 100 <= w128 * 115) bn = 256;  // BN = 256 has the more efficient main loop
+    // BN = 256 has the more efficient main loop, but a short-K residual GEMM is
+    // bound by its fp32 read-modify-write epilogue, which narrower tiles spread
+    // over more CTAs.
+    const bool short_resid = epi.mode == LAZYMAR_EPI_RESIDUAL && K < 2048;
+    if (!short_resid && w256 * 100 <= w128 * 115) bn = 256;
   }
   return bn == 256 ? launch_tc<256>(c, A, W, M, N, K, epi) : launch_tc<128>(c, A, W, M, N, K, epi);
 }

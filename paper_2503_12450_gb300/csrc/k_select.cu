@@ -12,7 +12,7 @@
 //
 // topk_kernel: one CTA per row. Each token's rank under the strict total order
 // (S ascending, index ascending; NaN counted as -inf) is counted against all T
-// similarities held in shared memory; tokens with rank < N are I_compute. A
+// similarities held in shared memory as order-preserving integer keys; tokens with rank < N are I_compute. A
 // block-wide ballot/prefix scan writes them in ascending index order together
 // with the gather/scatter row map r*T + t.
 #include <cfloat>
@@ -71,25 +71,34 @@ cudaError_t launch_similarity(const Ctx& c, int dtype, const void* cur, void* ca
 
 constexpr int kTopkThreads = 512;
 
+// Order-preserving 64-bit key of a similarity: unsigned comparison of keys
+// matches numeric comparison of the doubles, with NaN mapped to -inf and -0
+// to +0 (so equal similarities give equal keys and the index decides). Keys
+// are compared on the integer pipe; GB300's fp64 pipe is far slower.
+__device__ __forceinline__ unsigned long long sim_key(double s) {
+  if (s != s) s = -HUGE_VAL;
+  if (s == 0.0) s = 0.0;
+  const unsigned long long u = (unsigned long long)__double_as_longlong(s);
+  return (u >> 63) ? ~u : (u | 0x8000000000000000ull);
+}
+
 __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const double* __restrict__ S, int T, int N,
                                                             int* __restrict__ idx, int* __restrict__ row_map) {
-  extern __shared__ double sS[];  // T keys
+  extern __shared__ unsigned long long sK[];  // T keys
   __shared__ int s_wcount[kTopkThreads / 32];
   __shared__ int s_woff[kTopkThreads / 32];
   __shared__ int s_total;
-  unsigned char* sel = reinterpret_cast<unsigned char*>(sS + T);
+  unsigned char* sel = reinterpret_cast<unsigned char*>(sK + T);
   const int r = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  for (int t = tid; t < T; t += kTopkThreads) {
-    const double s = S[(size_t)r * T + t];
-    sS[t] = (s != s) ? -DBL_MAX * 2.0 : s;  // NaN -> -inf
-  }
+  for (int t = tid; t < T; t += kTopkThreads) sK[t] = sim_key(S[(size_t)r * T + t]);
   __syncthreads();
+  // rank of token t under (S ascending, index ascending); I_compute = rank < N
   for (int t = tid; t < T; t += kTopkThreads) {
-    const double st = sS[t];
+    const unsigned long long kt = sK[t];
     int rank = 0;
     for (int u = 0; u < T; ++u) {
-      const double su = sS[u];
-      rank += (su < st) || (su == st && u < t);
+      const unsigned long long ku = sK[u];
+      rank += (ku < kt) || (ku == kt && u < t);
     }
     sel[t] = rank < N;
   }
@@ -125,7 +134,7 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const double* __rest
 
 cudaError_t launch_topk(const Ctx& c, const double* S, int rows, int T, int N, int* idx, int* row_map) {
   if (rows == 0 || N == 0) return cudaSuccess;
-  const size_t smem = (size_t)T * sizeof(double) + (size_t)T;
+  const size_t smem = (size_t)T * sizeof(unsigned long long) + (size_t)T;
   if (smem > 48 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;

@@ -179,3 +179,17 @@ def test_layernorm(M, D, gather, dtype):
     sync()
     src = x[rm] if gather else x[:M]
     assert max_rel(host(y), O.layer_norm(src, g, b, 1e-6)) < (1e-2 if dtype == "bf16" else 1e-5)
+
+
+def test_gelu_epilogue_matches_erf_gelu():
+    """The MLP epilogue's GELU (erf from Abramowitz & Stegun 7.1.26, |error| <=
+    1.5e-7) against the oracle's fp64 erf GELU. An fp32 GEMM with W = I makes the
+    pre-activation exactly the input, on a dense grid over [-8, 8]."""
+    M, K = 512, 64
+    x = np.linspace(-8.0, 8.0, M * K, dtype=np.float32).reshape(M, K)
+    out = empty((M, K), "fp32")
+    lm.lazymar_linear(DT["fp32"], lm.LAZYMAR_EPI_GELU, dev(x), dev(np.eye(K, dtype=np.float32)), None, M, K, K,
+                      out, K)
+    sync()
+    err = np.abs(host(out) - O.gelu(x.astype(np.float64)))
+    assert (err <= 1e-6 * np.maximum(1.0, np.abs(x))).all(), float(err.max())
