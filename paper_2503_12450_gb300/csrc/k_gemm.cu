@@ -74,14 +74,27 @@ constexpr int BK = 64;   // one 128-byte swizzle atom of bf16 along K
 constexpr int kEpiWarps = 8;
 constexpr int kThreads = 64 + kEpiWarps * 32;
 
-template <int BN>
+// Epilogue kinds: BF16OUT stores bf16 (bias / GELU / Q-K-V split); the two
+// residual kinds add into the fp32 residual stream. RESID_WIDE stages whole
+// 32-column fp32 chunks (for short K, where the epilogue bounds the kernel, at
+// the cost of one pipeline stage); RESID_HALF stages 16-column halves and keeps
+// every stage (for long K, where the main loop bounds it).
+enum EpiKind { BF16OUT = 0, RESID_WIDE = 1, RESID_HALF = 2 };
+
+template <int BN, int EK>
 struct Cfg {
-  static constexpr int STAGES = (BN == 256) ? 4 : 6;
+  static constexpr int STAGES = EK == RESID_WIDE ? (BN == 256 ? 3 : 5) : (BN == 256 ? 4 : 6);
   static constexpr uint32_t A_BYTES = BM * BK * 2;
   static constexpr uint32_t B_BYTES = BN * BK * 2;
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulator buffers
-  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + 256;
+  // Per-warp staging of 32 rows (64 or 128 bytes each), rows padded by 16
+  // bytes so that both the row-wise writes and the column-block reads are
+  // bank-conflict-lean.
+  static constexpr uint32_t ROW_BYTES = EK == RESID_WIDE ? 128 : 64;
+  static constexpr uint32_t STG_PITCH = ROW_BYTES + 16;
+  static constexpr uint32_t STG_BYTES = 32 * STG_PITCH;
+  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + kEpiWarps * STG_BYTES + 256;
   // Instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1),
   // B bf16 (bits 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
   static constexpr uint32_t IDESC =
@@ -96,18 +109,31 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
   return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
          ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
+
+// Destination row pointer of a bf16 epilogue for tile row `row`, column `col`
+// (a 32-column chunk never straddles the Q/K/V parts).
+__device__ __forceinline__ bf16* out_row(const GemmEpi& e, int row, int col) {
+  if (e.mode != LAZYMAR_EPI_QKV) return static_cast<bf16*>(e.out) + (size_t)row * e.ldo + col;
+  const int part = col / e.D;
+  const int c = col - part * e.D;
+  if (part == 0) return static_cast<bf16*>(e.out) + (size_t)row * e.D + c;
+  const int drow = e.row_map ? e.row_map[row] : row;
+  return static_cast<bf16*>(part == 1 ? e.k_out : e.v_out) + (size_t)drow * e.D + c;
+}
 }  // namespace tc
 
-template <int BN>
+template <int BN, int EK>
 __global__ void __launch_bounds__(tc::kThreads, 1)
     gemm_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M,
                         int N, int K, GemmEpi epi, unsigned* err) {
-  using C = tc::Cfg<BN>;
+  using C = tc::Cfg<BN, EK>;
+  constexpr bool RESID = EK != tc::BF16OUT;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + C::STAGES * C::A_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  uint8_t* sStg = smem + C::STAGES * C::STAGE_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sStg + tc::kEpiWarps * C::STG_BYTES);
   uint64_t* empty = full + C::STAGES;
   uint64_t* acc_full = empty + C::STAGES;
   uint64_t* acc_empty = acc_full + 2;
@@ -190,56 +216,159 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
     __syncwarp();
   } else {
     // ---------------- epilogue warps ----------------
-    // The fp32 residual of a chunk does not depend on the accumulator, so the
-    // first chunk's residual is loaded before waiting for the accumulator and
-    // each later chunk's while the previous one is processed: the global-load
-    // latency overlaps the main loop instead of stalling the epilogue.
+    // Each warp owns 32 accumulator rows (its TMEM lane quarter) and half of
+    // the tile's columns, processed as 32 x 32 chunks. tcgen05.ld gives one row
+    // per thread; each chunk is transposed through the warp's staging buffer
+    // (32 rows x 64 bytes: 32 bf16 columns, or 16 fp32 columns at a time) so
+    // that every global store and residual load covers 8 rows x 64 contiguous
+    // bytes per warp instruction. The residual of the next chunk is loaded
+    // while the current one is processed, and the first chunk's before the
+    // accumulator is ready.
     const int ew = warp - 2;        // 0..7
     const int quarter = warp & 3;   // tensor-memory lanes this warp may read
     const int half = ew >> 2;       // which half of the tile's columns
     constexpr int CHUNKS = BN / 64; // 32-column chunks per half
-    const bool resid = epi.mode == LAZYMAR_EPI_RESIDUAL;
+    uint8_t* stg = sStg + ew * C::STG_BYTES;
+    const int cr = lane >> 2;       // row within an 8-row pass
+    const int cq = lane & 3;        // 16-byte block within the 64-byte row segment
     float* const res_base = static_cast<float*>(epi.out);
     int it = 0;
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++it) {
       const int buf = it & 1;
       const uint32_t use = (uint32_t)(it >> 1) & 1u;
       const int m0 = (tile % num_m) * tc::BM, n0 = (tile / num_m) * BN;
-      const int row = m0 + quarter * 32 + lane;
-      const bool row_ok = row < M;
+      const int rbase = m0 + quarter * 32;  // first of this warp's 32 rows
       const int c0 = half * CHUNKS;
-      float nxt[32];
-      if (resid && row_ok) Vec<float, 32>::load(res_base + (size_t)row * epi.ldo + n0 + c0 * 32, nxt);
+      // residual of a 32-column chunk in the coalesced layout: [16-col half][pass]
+      float4 res[2][4];
+      auto load_res = [&](int col) {
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+          for (int p = 0; p < 4; ++p) {
+            const int row = rbase + p * 8 + cr;
+            res[h][p] = row < M ? *reinterpret_cast<const float4*>(res_base + (size_t)row * epi.ldo + col + h * 16 + cq * 4)
+                                : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+      };
+      // RESID_WIDE layout: [pass] with 4 rows x 8 blocks of 16 bytes per pass
+      float4 resw[8];
+      auto load_resw = [&](int col) {
+        const int wr = lane >> 3, wq = lane & 7;
+#pragma unroll
+        for (int p = 0; p < 8; ++p) {
+          const int row = rbase + p * 4 + wr;
+          resw[p] = row < M ? *reinterpret_cast<const float4*>(res_base + (size_t)row * epi.ldo + col + wq * 4)
+                            : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      };
+      if (EK == tc::RESID_HALF) load_res(n0 + c0 * 32);
+      if (EK == tc::RESID_WIDE) load_resw(n0 + c0 * 32);
       const bool ok = mbar_wait(&acc_full[buf], use, abort_flag, err);
       if (__any_sync(0xffffffffu, !ok)) break;
       tc_fence_after();
 #pragma unroll 1
       for (int c = c0; c < c0 + CHUNKS; ++c) {
         const int col = n0 + c * 32;
-        float res[32];
-        if (resid) {
-#pragma unroll
-          for (int i = 0; i < 32; ++i) res[i] = nxt[i];
-          if (row_ok && c + 1 < c0 + CHUNKS) Vec<float, 32>::load(res_base + (size_t)row * epi.ldo + col + 32, nxt);
-        }
         uint32_t r[32];
         tmem_ld32(tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN + c * 32), r);
-        float bv[32];
-        if (epi.bias) Vec<bf16, 32>::load(static_cast<const bf16*>(epi.bias) + col, bv);
         tmem_wait_ld();
-        if (row_ok) {
+        if (EK == tc::RESID_WIDE) {
+          // whole 32-column fp32 chunk: 4 rows x 128 B per warp instruction
+          float4* srow = reinterpret_cast<float4*>(stg + lane * C::STG_PITCH);
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            srow[j] = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                                  __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+          __syncwarp();
+          const int wr = lane >> 3, wq = lane & 7;
+          float4 bq = make_float4(0.f, 0.f, 0.f, 0.f);
+          if (epi.bias) {
+            float bv[8];
+            Vec<bf16, 8>::load(static_cast<const bf16*>(epi.bias) + col + (wq & ~1) * 4, bv);
+            const int o = (wq & 1) * 4;
+            bq = make_float4(bv[o], bv[o + 1], bv[o + 2], bv[o + 3]);
+          }
+          float4 cur[8];
+#pragma unroll
+          for (int p = 0; p < 8; ++p) cur[p] = resw[p];
+          if (c + 1 < c0 + CHUNKS) load_resw(col + 32);  // prefetch the next chunk
+#pragma unroll
+          for (int p = 0; p < 8; ++p) {
+            const int lr = p * 4 + wr;
+            const int row = rbase + lr;
+            const float4 a = *reinterpret_cast<const float4*>(stg + lr * C::STG_PITCH + wq * 16);
+            if (row < M) {
+              float4 o;
+              o.x = cur[p].x + (a.x + bq.x);
+              o.y = cur[p].y + (a.y + bq.y);
+              o.z = cur[p].z + (a.z + bq.z);
+              o.w = cur[p].w + (a.w + bq.w);
+              *reinterpret_cast<float4*>(res_base + (size_t)row * epi.ldo + col + wq * 4) = o;
+            }
+          }
+          __syncwarp();
+        } else if (EK == tc::RESID_HALF) {
+          float4 cur[2][4];
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int p = 0; p < 4; ++p) cur[h][p] = res[h][p];
+          if (c + 1 < c0 + CHUNKS) load_res(col + 32);  // prefetch the next chunk
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            // stage 16 raw fp32 accumulator columns of this thread's row
+            float4* srow = reinterpret_cast<float4*>(stg + lane * C::STG_PITCH);
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              srow[j] = make_float4(__uint_as_float(r[16 * h + 4 * j]), __uint_as_float(r[16 * h + 4 * j + 1]),
+                                    __uint_as_float(r[16 * h + 4 * j + 2]), __uint_as_float(r[16 * h + 4 * j + 3]));
+            __syncwarp();
+            float4 bq = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (epi.bias) {
+              float bv[8];
+              Vec<bf16, 8>::load(static_cast<const bf16*>(epi.bias) + col + h * 16 + (cq & ~1) * 4, bv);
+              const int o = (cq & 1) * 4;
+              bq = make_float4(bv[o], bv[o + 1], bv[o + 2], bv[o + 3]);
+            }
+#pragma unroll
+            for (int p = 0; p < 4; ++p) {
+              const int lr = p * 8 + cr;
+              const int row = rbase + lr;
+              const float4 a = *reinterpret_cast<const float4*>(stg + lr * C::STG_PITCH + cq * 16);
+              if (row < M) {
+                float4 o;
+                o.x = cur[h][p].x + (a.x + bq.x);
+                o.y = cur[h][p].y + (a.y + bq.y);
+                o.z = cur[h][p].z + (a.z + bq.z);
+                o.w = cur[h][p].w + (a.w + bq.w);
+                *reinterpret_cast<float4*>(res_base + (size_t)row * epi.ldo + col + h * 16 + cq * 4) = o;
+              }
+            }
+            __syncwarp();
+          }
+        } else {
+          // bias (+ GELU) in the row layout, bf16 to the staging buffer, then
+          // whole-row-segment stores
+          float bv[32];
+          if (epi.bias) Vec<bf16, 32>::load(static_cast<const bf16*>(epi.bias) + col, bv);
           float v[32];
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]) + (epi.bias ? bv[i] : 0.f);
-          if (resid) {
+          if (epi.mode == LAZYMAR_EPI_GELU) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] += res[i];
-            Vec<float, 32>::store(res_base + (size_t)row * epi.ldo + col, v);
-          } else {
-            GemmEpi e2 = epi;
-            e2.bias = nullptr;
-            epilogue_apply<bf16, 32>(e2, row, col, v);
+            for (int i = 0; i < 32; ++i) v[i] = gelu_erf(v[i]);
           }
+          Vec<bf16, 32>::store(reinterpret_cast<bf16*>(stg + lane * C::STG_PITCH), v);
+          __syncwarp();
+#pragma unroll
+          for (int p = 0; p < 4; ++p) {
+            const int lr = p * 8 + cr;
+            const int row = rbase + lr;
+            const uint4 val = *reinterpret_cast<const uint4*>(stg + lr * C::STG_PITCH + cq * 16);
+            if (row < M) *reinterpret_cast<uint4*>(tc::out_row(epi, row, col) + cq * 8) = val;
+          }
+          __syncwarp();
         }
       }
       tc_fence_before();
@@ -348,9 +477,9 @@ bool gemm_supported(int dtype, int M, int N, int K, const GemmEpi& epi, const ch
   return true;
 }
 
-template <int BN>
+template <int BN, int EK>
 static cudaError_t launch_tc(const Ctx& c, const void* A, const void* W, int M, int N, int K, const GemmEpi& epi) {
-  using C = tc::Cfg<BN>;
+  using C = tc::Cfg<BN, EK>;
   CUtensorMap ta, tb;
   if (!make_tmap_bf16(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * 2, tc::BK, tc::BM,
                       CU_TENSOR_MAP_SWIZZLE_128B) ||
@@ -360,14 +489,14 @@ static cudaError_t launch_tc(const Ctx& c, const void* A, const void* W, int M, 
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc_kernel<BN, EK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)C::SMEM);
     if (e != cudaSuccess) return e;
     attr_set[dev] = 1;
   }
   const int tiles = ((M + tc::BM - 1) / tc::BM) * (N / BN);
   const int grid = tiles < c.num_sms ? tiles : c.num_sms;
-  gemm_bf16_tc_kernel<BN><<<grid, tc::kThreads, C::SMEM, c.stream>>>(ta, tb, M, N, K, epi, c.err);
+  gemm_bf16_tc_kernel<BN, EK><<<grid, tc::kThreads, C::SMEM, c.stream>>>(ta, tb, M, N, K, epi, c.err);
   return cudaGetLastError();
 }
 
@@ -386,15 +515,22 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
     bn = 256;
   } else if (flags == 0 && N % 256 == 0) {
     const long mt = (M + tc::BM - 1) / tc::BM;
-    const long w128 = (mt * (N / 128) + c.num_sms - 1) / c.num_sms * 128;
-    const long w256 = (mt * (N / 256) + c.num_sms - 1) / c.num_sms * 256;
-    // BN = 256 has the more efficient main loop, but a short-K residual GEMM is
-    // bound by its fp32 read-modify-write epilogue, which narrower tiles spread
-    // over more CTAs.
-    const bool short_resid = epi.mode == LAZYMAR_EPI_RESIDUAL && K < 2048;
-    if (!short_resid && w256 * 100 <= w128 * 115) bn = 256;
+    const long w128 = (mt * (N / 128) + c.num_sms - 1) / c.num_sms;  // waves of BN = 128 tiles
+    const long w256 = (mt * (N / 256) + c.num_sms - 1) / c.num_sms;  // waves of BN = 256 tiles
+    // A BN = 128 tile is capped by shared-memory bandwidth at about 0.56x the
+    // main-loop rate of a BN = 256 tile (measured), so BN = 256 wins unless it
+    // leaves more than 1.12x as many tile-waves idle.
+    if (w256 * 112 <= w128 * 100) bn = 256;
   }
-  return bn == 256 ? launch_tc<256>(c, A, W, M, N, K, epi) : launch_tc<128>(c, A, W, M, N, K, epi);
+  const int ek = epi.mode != LAZYMAR_EPI_RESIDUAL ? tc::BF16OUT : (K < 2048 ? tc::RESID_WIDE : tc::RESID_HALF);
+  if (bn == 256) {
+    if (ek == tc::RESID_WIDE) return launch_tc<256, tc::RESID_WIDE>(c, A, W, M, N, K, epi);
+    if (ek == tc::RESID_HALF) return launch_tc<256, tc::RESID_HALF>(c, A, W, M, N, K, epi);
+    return launch_tc<256, tc::BF16OUT>(c, A, W, M, N, K, epi);
+  }
+  if (ek == tc::RESID_WIDE) return launch_tc<128, tc::RESID_WIDE>(c, A, W, M, N, K, epi);
+  if (ek == tc::RESID_HALF) return launch_tc<128, tc::RESID_HALF>(c, A, W, M, N, K, epi);
+  return launch_tc<128, tc::BF16OUT>(c, A, W, M, N, K, epi);
 }
 
 }  // namespace lm
