@@ -18,46 +18,86 @@ namespace lm {
 // ---------------------------------------------------------------------------
 // Embedding
 // ---------------------------------------------------------------------------
+// One thread per (token, 4 consecutive columns), grid-stride; the 16-float
+// latent of a decoded token is read by all threads of that token (L1 hits).
 template <typename TW>
+__device__ __forceinline__ float4 load4(const TW* p) {
+  if constexpr (sizeof(TW) == 2) {
+    const uint2 u = *reinterpret_cast<const uint2*>(p);
+    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+    const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+    return make_float4(a.x, a.y, b.x, b.y);
+  } else {
+    return *reinterpret_cast<const float4*>(p);
+  }
+}
+
+template <typename TW, int TD>
 __global__ void __launch_bounds__(256) embed_kernel(const float* __restrict__ lat, const uint8_t* __restrict__ mask,
                                                     const int* __restrict__ labels, const TW* __restrict__ pos,
                                                     const TW* __restrict__ cls, const TW* __restrict__ memb,
                                                     const TW* __restrict__ ew, const TW* __restrict__ eb,
-                                                    float* __restrict__ H, int B, int T, int nb, int n_img, int D,
-                                                    int tdim, int n_classes, unsigned* err) {
-  __shared__ float sl[64];
-  const int tok = blockIdx.x;  // r * T + t
-  const int r = tok / T, t = tok - r * T;
-  const bool cond = r < B;
-  const int pair = cond ? r : r - B;
-  float* out = H + (size_t)tok * D;
-  const TW* p = pos + (size_t)t * D;
-  if (t < nb) {
-    const TW* c = nullptr;
-    if (cond) {
-      int y = labels[pair];
-      if (y < 0 || y >= n_classes) {
-        if (threadIdx.x == 0) atomicOr(err, ERR_LABEL);
-        y = 0;
+                                                    float* __restrict__ H, int n4, int B, int T, int nb, int n_img,
+                                                    int D, int tdim, int n_classes, unsigned* err) {
+  const int D4 = D / 4;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += gridDim.x * blockDim.x) {
+    const int tok = i / D4;  // r * T + t
+    const int d = (i - tok * D4) * 4;
+    const int r = tok / T, t = tok - r * T;
+    const bool cond = r < B;
+    const int pair = cond ? r : r - B;
+    float4 v = load4(pos + (size_t)t * D + d);
+    if (t < nb) {
+      if (cond) {
+        int y = labels[pair];
+        if (y < 0 || y >= n_classes) {
+          if (d == 0) atomicOr(err, ERR_LABEL);
+          y = 0;
+        }
+        const float4 c = load4(cls + (size_t)y * D + d);
+        v.x += c.x; v.y += c.y; v.z += c.z; v.w += c.w;
       }
-      c = cls + (size_t)y * D;
+    } else {
+      const int img = t - nb;
+      if (mask[(size_t)pair * n_img + img]) {
+        const float4 m = load4(memb + d);
+        v.x += m.x; v.y += m.y; v.z += m.z; v.w += m.w;
+      } else {
+        const float* lr = lat + ((size_t)pair * n_img + img) * tdim;
+        const float4 bb = load4(eb + d);
+        float acc[4] = {bb.x, bb.y, bb.z, bb.w};
+        if constexpr (TD > 0) {
+          // latent width known at compile time: vector loads of the latent
+          // and of each of the 4 weight rows (TD contiguous values)
+          float l[TD > 0 ? TD : 4];
+#pragma unroll
+          for (int j = 0; j < TD; j += 4) {
+            const float4 q = *reinterpret_cast<const float4*>(lr + j);
+            l[j] = q.x; l[j + 1] = q.y; l[j + 2] = q.z; l[j + 3] = q.w;
+          }
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const TW* w = ew + (size_t)(d + k) * TD;
+#pragma unroll
+            for (int j = 0; j < TD; j += 4) {
+              const float4 wq = load4(w + j);
+              acc[k] = fmaf(wq.x, l[j], acc[k]);
+              acc[k] = fmaf(wq.y, l[j + 1], acc[k]);
+              acc[k] = fmaf(wq.z, l[j + 2], acc[k]);
+              acc[k] = fmaf(wq.w, l[j + 3], acc[k]);
+            }
+          }
+        } else {
+          for (int j = 0; j < tdim; ++j) {
+            const float lj = lr[j];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) acc[k] = fmaf(to_f(ew[(size_t)(d + k) * tdim + j]), lj, acc[k]);
+          }
+        }
+        v.x += acc[0]; v.y += acc[1]; v.z += acc[2]; v.w += acc[3];
+      }
     }
-    for (int d = threadIdx.x; d < D; d += blockDim.x) out[d] = to_f(p[d]) + (c ? to_f(c[d]) : 0.f);
-    return;
-  }
-  const int i = t - nb;
-  if (mask[(size_t)pair * n_img + i]) {
-    for (int d = threadIdx.x; d < D; d += blockDim.x) out[d] = to_f(p[d]) + to_f(memb[d]);
-    return;
-  }
-  const float* lr = lat + ((size_t)pair * n_img + i) * tdim;
-  for (int j = threadIdx.x; j < tdim; j += blockDim.x) sl[j] = lr[j];
-  __syncthreads();
-  for (int d = threadIdx.x; d < D; d += blockDim.x) {
-    const TW* w = ew + (size_t)d * tdim;
-    float acc = to_f(eb[d]);
-    for (int j = 0; j < tdim; ++j) acc = fmaf(to_f(w[j]), sl[j], acc);
-    out[d] = to_f(p[d]) + acc;
+    *reinterpret_cast<float4*>(H + (size_t)tok * D + d) = v;
   }
 }
 
@@ -65,15 +105,22 @@ cudaError_t launch_embed(const Ctx& c, int dtype, const float* lat, const uint8_
                          const void* pos, const void* cls, const void* memb, const void* ew, const void* eb, float* H,
                          int rows, int B, int T, int nb, int n_img, int D, int tdim, int n_classes) {
   if (rows == 0) return cudaSuccess;
-  const unsigned grid = (unsigned)(rows * T);
-  if (dtype == LAZYMAR_BF16)
-    embed_kernel<bf16><<<grid, 256, 0, c.stream>>>(lat, mask, labels, (const bf16*)pos, (const bf16*)cls,
-                                                   (const bf16*)memb, (const bf16*)ew, (const bf16*)eb, H, B, T, nb,
-                                                   n_img, D, tdim, n_classes, c.err);
-  else
-    embed_kernel<float><<<grid, 256, 0, c.stream>>>(lat, mask, labels, (const float*)pos, (const float*)cls,
-                                                    (const float*)memb, (const float*)ew, (const float*)eb, H, B, T,
-                                                    nb, n_img, D, tdim, n_classes, c.err);
+  const long long n4l = (long long)rows * T * (D / 4);
+  if (n4l >= (1ll << 31)) return cudaErrorInvalidValue;
+  const int n4 = (int)n4l;
+  long long blocks = (n4l + 255) / 256;
+  const long long cap = (long long)c.num_sms * 16;
+  if (blocks > cap) blocks = cap;
+#define LM_EMBED(TW, TD)                                                                                      \
+  embed_kernel<TW, TD><<<(unsigned)blocks, 256, 0, c.stream>>>(                                              \
+      lat, mask, labels, (const TW*)pos, (const TW*)cls, (const TW*)memb, (const TW*)ew, (const TW*)eb, H, n4, B, \
+      T, nb, n_img, D, tdim, n_classes, c.err)
+  if (dtype == LAZYMAR_BF16) {
+    if (tdim == 16) LM_EMBED(bf16, 16); else LM_EMBED(bf16, 0);
+  } else {
+    if (tdim == 16) LM_EMBED(float, 16); else LM_EMBED(float, 0);
+  }
+#undef LM_EMBED
   return cudaGetLastError();
 }
 
