@@ -78,6 +78,8 @@ __global__ void __launch_bounds__(128) attention_bf16_kernel(const __grid_consta
     fence_mbar_init();
   }
   __syncthreads();
+  pdl_wait();
+  pdl_trigger();
   if (tid == 0) {
     mbar_arrive_expect_tx(&bars[0], q_bytes);
     tma_load_2d(&tmQ, &bars[0], sQ, col, q0);
@@ -229,6 +231,8 @@ __global__ void __launch_bounds__(128) attention_f32_kernel(const float* __restr
                                                             const float* __restrict__ v, float* __restrict__ o,
                                                             int n_q, int T, int D, int dh, float scale) {
   extern __shared__ float sm[];
+  pdl_wait();
+  pdl_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   float* sc = sm + warp * (T + dh);
   float* qv = sc + T;
@@ -305,9 +309,8 @@ static cudaError_t launch_attn_bf16(const Ctx& c, const void* q, const void* k, 
   }
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
   dim3 grid((n_q + at::QT - 1) / at::QT, heads, rows);
-  attention_bf16_kernel<DH><<<grid, 128, smem, c.stream>>>(mq, mq2, mk, mk2, mv, mv2, static_cast<bf16*>(o), n_q,
-                                                           T, D, scale_log2, c.err);
-  return cudaGetLastError();
+  return launch_pdl(attention_bf16_kernel<DH>, grid, dim3(128), smem, c.stream, mq, mq2, mk, mk2, mv, mv2,
+                    static_cast<bf16*>(o), n_q, T, D, scale_log2, c.err);
 }
 
 cudaError_t launch_attention(const Ctx& c, int dtype, const void* q, const void* k, const void* v, void* o,
@@ -321,10 +324,9 @@ cudaError_t launch_attention(const Ctx& c, int dtype, const void* q, const void*
       if (e != cudaSuccess) return e;
     }
     dim3 grid((n_q + 3) / 4, heads, rows);
-    attention_f32_kernel<<<grid, 128, smem, c.stream>>>(static_cast<const float*>(q), static_cast<const float*>(k),
-                                                        static_cast<const float*>(v), static_cast<float*>(o), n_q, T,
-                                                        heads * dh, dh, 1.0f / sqrtf((float)dh));
-    return cudaGetLastError();
+    return launch_pdl(attention_f32_kernel, grid, dim3(128), smem, c.stream, static_cast<const float*>(q),
+                      static_cast<const float*>(k), static_cast<const float*>(v), static_cast<float*>(o), n_q, T,
+                      heads * dh, dh, 1.0f / sqrtf((float)dh));
   }
   if (dh == 64) return launch_attn_bf16<64>(c, q, k, v, o, rows, n_q, T, heads);
   return launch_attn_bf16<80>(c, q, k, v, o, rows, n_q, T, heads);

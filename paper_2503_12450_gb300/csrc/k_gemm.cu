@@ -167,6 +167,20 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // Weights are never written by any kernel, so the producer fetches the
+  // weight tiles of its first stages before waiting for the predecessor grid;
+  // every other access follows pdl_wait().
+  int pre = 0;
+  if (warp == 0 && lane == 0 && (int)blockIdx.x < tiles) {
+    const int n0 = ((int)blockIdx.x / num_m) * BN;
+    pre = KB < C::STAGES ? KB : C::STAGES;
+    for (int s = 0; s < pre; ++s) {
+      mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
+      tma_load_2d(&tmB, &full[s], sB + s * C::B_BYTES, s * tc::BK, n0);
+    }
+  }
+  pdl_wait();
+  pdl_trigger();
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
@@ -177,10 +191,15 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
       for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
         const int m0 = (tile % num_m) * tc::BM, n0 = (tile / num_m) * BN;
         for (int kb = 0; kb < KB; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
-          mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
-          tma_load_2d(&tmA, &full[stage], sA + stage * C::A_BYTES, kb * tc::BK, m0);
-          tma_load_2d(&tmB, &full[stage], sB + stage * C::B_BYTES, kb * tc::BK, n0);
+          if (tile == (int)blockIdx.x && kb < pre) {
+            // weight tile already in flight on this stage: add the activations
+            tma_load_2d(&tmA, &full[stage], sA + stage * C::A_BYTES, kb * tc::BK, m0);
+          } else {
+            if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
+            mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
+            tma_load_2d(&tmA, &full[stage], sA + stage * C::A_BYTES, kb * tc::BK, m0);
+            tma_load_2d(&tmB, &full[stage], sB + stage * C::B_BYTES, kb * tc::BK, n0);
+          }
           if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
         }
       }
@@ -390,6 +409,8 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(const float* __restrict__
                                                        int N, int K, GemmEpi epi) {
   __shared__ float As[16][64 + 4];
   __shared__ float Ws[16][64 + 4];
+  pdl_wait();
+  pdl_trigger();
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
   const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
   float acc[4][4] = {};
@@ -496,8 +517,8 @@ static cudaError_t launch_tc(const Ctx& c, const void* A, const void* W, int M, 
   }
   const int tiles = ((M + tc::BM - 1) / tc::BM) * (N / BN);
   const int grid = tiles < c.num_sms ? tiles : c.num_sms;
-  gemm_bf16_tc_kernel<BN, EK><<<grid, tc::kThreads, C::SMEM, c.stream>>>(ta, tb, M, N, K, epi, c.err);
-  return cudaGetLastError();
+  return launch_pdl(gemm_bf16_tc_kernel<BN, EK>, dim3(grid), dim3(tc::kThreads), C::SMEM, c.stream, ta, tb, M, N, K,
+                    epi, c.err);
 }
 
 cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, int M, int N, int K,
@@ -505,9 +526,8 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
   if (M == 0) return cudaSuccess;
   if (dtype == LAZYMAR_F32) {
     dim3 grid((N + 63) / 64, (M + 63) / 64);
-    gemm_f32_kernel<<<grid, 256, 0, c.stream>>>(static_cast<const float*>(A), static_cast<const float*>(W), M, N,
-                                                 K, epi);
-    return cudaGetLastError();
+    return launch_pdl(gemm_f32_kernel, grid, dim3(256), 0, c.stream, static_cast<const float*>(A),
+                      static_cast<const float*>(W), M, N, K, epi);
   }
   // Tile width: the one with fewer tile-waves x tile-time over the SMs.
   int bn = 128;

@@ -40,6 +40,8 @@ __global__ void __launch_bounds__(256) embed_kernel(const float* __restrict__ la
                                                     float* __restrict__ H, int n4, int B, int T, int nb, int n_img,
                                                     int D, int tdim, int n_classes, unsigned* err) {
   const int D4 = D / 4;
+  pdl_wait();
+  pdl_trigger();
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += gridDim.x * blockDim.x) {
     const int tok = i / D4;  // r * T + t
     const int d = (i - tok * D4) * 4;
@@ -111,17 +113,13 @@ cudaError_t launch_embed(const Ctx& c, int dtype, const float* lat, const uint8_
   long long blocks = (n4l + 255) / 256;
   const long long cap = (long long)c.num_sms * 16;
   if (blocks > cap) blocks = cap;
-#define LM_EMBED(TW, TD)                                                                                      \
-  embed_kernel<TW, TD><<<(unsigned)blocks, 256, 0, c.stream>>>(                                              \
-      lat, mask, labels, (const TW*)pos, (const TW*)cls, (const TW*)memb, (const TW*)ew, (const TW*)eb, H, n4, B, \
-      T, nb, n_img, D, tdim, n_classes, c.err)
-  if (dtype == LAZYMAR_BF16) {
-    if (tdim == 16) LM_EMBED(bf16, 16); else LM_EMBED(bf16, 0);
-  } else {
-    if (tdim == 16) LM_EMBED(float, 16); else LM_EMBED(float, 0);
-  }
+#define LM_EMBED(TW, TD)                                                                                    \
+  launch_pdl(embed_kernel<TW, TD>, dim3((unsigned)blocks), dim3(256), 0, c.stream, lat, mask, labels,        \
+             (const TW*)pos, (const TW*)cls, (const TW*)memb, (const TW*)ew, (const TW*)eb, H, n4, B, T, nb, \
+             n_img, D, tdim, n_classes, c.err)
+  if (dtype == LAZYMAR_BF16) return tdim == 16 ? LM_EMBED(bf16, 16) : LM_EMBED(bf16, 0);
+  return tdim == 16 ? LM_EMBED(float, 16) : LM_EMBED(float, 0);
 #undef LM_EMBED
-  return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------------------
@@ -163,6 +161,8 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const float* __restrict_
                                                         const TO* __restrict__ g, const TO* __restrict__ b,
                                                         TO* __restrict__ y, float* __restrict__ x_copy, int M, int D,
                                                         float eps) {
+  pdl_wait();
+  pdl_trigger();
   const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (row >= M) return;
   const int src = row_map ? row_map[row] : row;
@@ -187,6 +187,8 @@ __global__ void __launch_bounds__(256) final_ln_kernel(const float* __restrict__
                                                        int T, int nb, int n_img, const TO* __restrict__ g,
                                                        const TO* __restrict__ b, TO* __restrict__ z, int M, int D,
                                                        float eps) {
+  pdl_wait();
+  pdl_trigger();
   const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (row >= M) return;
   const int tok = row_map ? row_map[row] : row;
@@ -203,17 +205,17 @@ __global__ void __launch_bounds__(256) final_ln_kernel(const float* __restrict__
   for (int i = 0; i < NV; ++i) ln_write4<TO>(zr, g, b, 4 * (lane + 32 * i), v[i], mean, rstd);
 }
 
-#define LM_LN_DISPATCH(KERNEL, TO, ...)                                                    \
-  switch (D / 128) {                                                                     \
-    case 1: KERNEL<TO, 1><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;               \
-    case 2: KERNEL<TO, 2><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;               \
-    case 4: KERNEL<TO, 4><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;               \
-    case 6: KERNEL<TO, 6><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;               \
-    case 8: KERNEL<TO, 8><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;               \
-    case 10: KERNEL<TO, 10><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;             \
-    case 12: KERNEL<TO, 12><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;             \
-    case 16: KERNEL<TO, 16><<<grid, 256, 0, c.stream>>>(__VA_ARGS__); break;             \
-    default: return cudaErrorInvalidValue;                                               \
+#define LM_LN_DISPATCH(KERNEL, TO, ...)                                                          \
+  switch (D / 128) {                                                                             \
+    case 1: return launch_pdl(KERNEL<TO, 1>, dim3(grid), dim3(256), 0, c.stream, __VA_ARGS__);   \
+    case 2: return launch_pdl(KERNEL<TO, 2>, dim3(grid), dim3(256), 0, c.stream, __VA_ARGS__);   \
+    case 4: return launch_pdl(KERNEL<TO, 4>, dim3(grid), dim3(256), 0, c.stream, __VA_ARGS__);   \
+    case 6: return launch_pdl(KERNEL<TO, 6>, dim3(grid), dim3(256), 0, c.stream, __VA_ARGS__);   \
+    case 8: return launch_pdl(KERNEL<TO, 8>, dim3(grid), dim3(256), 0, c.stream, __VA_ARGS__);   \
+    case 10: return launch_pdl(KERNEL<TO, 10>, dim3(grid), dim3(256), 0, c.stream, __VA_ARGS__); \
+    case 12: return launch_pdl(KERNEL<TO, 12>, dim3(grid), dim3(256), 0, c.stream, __VA_ARGS__); \
+    case 16: return launch_pdl(KERNEL<TO, 16>, dim3(grid), dim3(256), 0, c.stream, __VA_ARGS__); \
+    default: return cudaErrorInvalidValue;                                                       \
   }
 
 bool layernorm_width_ok(int D) {
@@ -252,17 +254,16 @@ cudaError_t launch_final_ln(const Ctx& c, int dtype, const float* x, const int* 
 // criterion when criterion == FEATURE).
 template <typename TO>
 __global__ void cast_kernel(const float* __restrict__ x, TO* __restrict__ y, size_t n) {
+  pdl_wait();
+  pdl_trigger();
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x)
     y[i] = from_f<TO>(x[i]);
 }
 cudaError_t launch_cast(const Ctx& c, int dtype, const float* x, void* y, size_t n) {
   if (n == 0) return cudaSuccess;
   const unsigned grid = (unsigned)((n + 255) / 256 < (size_t)c.num_sms * 8 ? (n + 255) / 256 : (size_t)c.num_sms * 8);
-  if (dtype == LAZYMAR_BF16)
-    cast_kernel<bf16><<<grid, 256, 0, c.stream>>>(x, (bf16*)y, n);
-  else
-    cast_kernel<float><<<grid, 256, 0, c.stream>>>(x, (float*)y, n);
-  return cudaGetLastError();
+  if (dtype == LAZYMAR_BF16) return launch_pdl(cast_kernel<bf16>, dim3(grid), dim3(256), 0, c.stream, x, (bf16*)y, n);
+  return launch_pdl(cast_kernel<float>, dim3(grid), dim3(256), 0, c.stream, x, (float*)y, n);
 }
 
 // ---------------------------------------------------------------------------
@@ -289,6 +290,8 @@ __global__ void __launch_bounds__(256) cfg_kernel(int mode, const T* __restrict_
                                                   T* __restrict__ delta, float gamma, size_t n, T* __restrict__ zu_out,
                                                   T* __restrict__ g_out) {
   constexpr int V = 16 / sizeof(T);
+  pdl_wait();
+  pdl_trigger();
   const size_t nv = n / V;
   const size_t stride = (size_t)gridDim.x * blockDim.x;
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < nv; i += stride) {
@@ -326,12 +329,10 @@ cudaError_t launch_cfg(const Ctx& c, int dtype, int mode, const void* zc, const 
   if (blocks > cap) blocks = cap;
   if (blocks == 0) blocks = 1;
   if (dtype == LAZYMAR_BF16)
-    cfg_kernel<bf16><<<(unsigned)blocks, 256, 0, c.stream>>>(mode, (const bf16*)zc, (const bf16*)zu, (bf16*)delta,
-                                                             gamma, n, (bf16*)zu_out, (bf16*)g_out);
-  else
-    cfg_kernel<float><<<(unsigned)blocks, 256, 0, c.stream>>>(mode, (const float*)zc, (const float*)zu,
-                                                              (float*)delta, gamma, n, (float*)zu_out, (float*)g_out);
-  return cudaGetLastError();
+    return launch_pdl(cfg_kernel<bf16>, dim3((unsigned)blocks), dim3(256), 0, c.stream, mode, (const bf16*)zc,
+                      (const bf16*)zu, (bf16*)delta, gamma, n, (bf16*)zu_out, (bf16*)g_out);
+  return launch_pdl(cfg_kernel<float>, dim3((unsigned)blocks), dim3(256), 0, c.stream, mode, (const float*)zc,
+                    (const float*)zu, (float*)delta, gamma, n, (float*)zu_out, (float*)g_out);
 }
 
 }  // namespace lm

@@ -26,6 +26,8 @@ template <typename T>
 __global__ void __launch_bounds__(256) similarity_kernel(const T* __restrict__ cur, T* __restrict__ cache,
                                                          double* __restrict__ S, long long ntok, int D, int copy) {
   constexpr int V = 16 / sizeof(T);
+  pdl_wait();
+  pdl_trigger();
   const long long tok = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (tok >= ntok) return;
@@ -63,10 +65,10 @@ cudaError_t launch_similarity(const Ctx& c, int dtype, const void* cur, void* ca
   if (ntok == 0) return cudaSuccess;
   const unsigned grid = (unsigned)((ntok + 7) / 8);
   if (dtype == LAZYMAR_BF16)
-    similarity_kernel<bf16><<<grid, 256, 0, c.stream>>>((const bf16*)cur, (bf16*)cache, S, ntok, D, copy ? 1 : 0);
-  else
-    similarity_kernel<float><<<grid, 256, 0, c.stream>>>((const float*)cur, (float*)cache, S, ntok, D, copy ? 1 : 0);
-  return cudaGetLastError();
+    return launch_pdl(similarity_kernel<bf16>, dim3(grid), dim3(256), 0, c.stream, (const bf16*)cur, (bf16*)cache, S,
+                      ntok, D, copy ? 1 : 0);
+  return launch_pdl(similarity_kernel<float>, dim3(grid), dim3(256), 0, c.stream, (const float*)cur, (float*)cache, S,
+                    ntok, D, copy ? 1 : 0);
 }
 
 constexpr int kTopkThreads = 512;
@@ -90,6 +92,8 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const double* __rest
   __shared__ int s_total;
   unsigned char* sel = reinterpret_cast<unsigned char*>(sK + T);
   const int r = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  pdl_wait();
+  pdl_trigger();
   for (int t = tid; t < T; t += kTopkThreads) sK[t] = sim_key(S[(size_t)r * T + t]);
   __syncthreads();
   // rank of token t under (S ascending, index ascending); I_compute = rank < N
@@ -139,8 +143,7 @@ cudaError_t launch_topk(const Ctx& c, const double* S, int rows, int T, int N, i
     cudaError_t e = cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
   }
-  topk_kernel<<<rows, kTopkThreads, smem, c.stream>>>(S, T, N, idx, row_map);
-  return cudaGetLastError();
+  return launch_pdl(topk_kernel, dim3(rows), dim3(kTopkThreads), smem, c.stream, S, T, N, idx, row_map);
 }
 
 // Caller-chosen I_compute: copied after checking range and strict increase per
@@ -148,6 +151,8 @@ cudaError_t launch_topk(const Ctx& c, const double* S, int rows, int T, int N, i
 // [0, T) so that no later gather or scatter leaves the row.
 __global__ void idx_check_kernel(const int* __restrict__ in, int rows, int T, int N, int* __restrict__ idx,
                                  int* __restrict__ row_map, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
   if (i >= (long long)rows * N) return;
   const int r = (int)(i / N), j = (int)(i - (long long)r * N);
@@ -164,8 +169,8 @@ __global__ void idx_check_kernel(const int* __restrict__ in, int rows, int T, in
 cudaError_t launch_idx_check(const Ctx& c, const int* in, int rows, int T, int N, int* idx, int* row_map) {
   const long long n = (long long)rows * N;
   if (n == 0) return cudaSuccess;
-  idx_check_kernel<<<(unsigned)((n + 255) / 256), 256, 0, c.stream>>>(in, rows, T, N, idx, row_map, c.err);
-  return cudaGetLastError();
+  return launch_pdl(idx_check_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, c.stream, in, rows, T, N, idx,
+                    row_map, c.err);
 }
 
 // ---------------------------------------------------------------------------

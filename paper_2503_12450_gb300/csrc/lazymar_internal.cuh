@@ -8,6 +8,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <utility>
 
 #include "../../include/lazymar.h"
 
@@ -129,6 +130,36 @@ template <int NC> struct Vec<float, NC> {
       reinterpret_cast<float4*>(p)[c] = make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
   }
 };
+
+// ---------------------------------------------------------------------------
+// Programmatic dependent launch
+// ---------------------------------------------------------------------------
+// Every kernel is launched so that it may start while its predecessor in the
+// stream drains: its CTAs can initialise barriers, allocate tensor memory and
+// prefetch descriptors early. pdl_wait() must precede the kernel's first access
+// to global memory that a predecessor writes or reads; it returns once the
+// predecessor grid has completed and its writes are visible. pdl_trigger()
+// allows the successor to be scheduled once every CTA of this grid has issued
+// it (so a successor never takes an SM a not-yet-started CTA of this grid
+// needs). Both are no-ops for a kernel launched without the attribute.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                              Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 // ---------------------------------------------------------------------------
 // Shared-memory barriers and TMA (PTX ISA: mbarrier, cp.async.bulk.tensor)
