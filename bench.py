@@ -56,16 +56,24 @@ def peaks():
     return dict(FALLBACK_PEAKS), "fallback"
 
 
+NAMES = {"mar_b": "MAR-B", "mar_l": "MAR-L", "mar_h": "MAR-H", "hires": "MAR-L high-resolution", "tiny": "tiny"}
+
+
 def workload(cfg):
     n = synth.n_compute(cfg)
     return {
-        "workload": "MAR-B-shaped 64-step LazyMAR decode (24 blocks, width 768, 12 heads, 64+256 tokens)",
+        "workload": "%s-shaped %d-step LazyMAR decode (%d blocks, width %d, %d heads, %d+%d tokens)" % (
+            NAMES.get(cfg["name"], cfg["name"]), cfg["steps"], cfg["depth"], cfg["width"], cfg["heads"],
+            cfg["n_buffer"], cfg["n_img"]),
         "batch_pairs": cfg["batch"], "rows": 2 * cfg["batch"], "tokens": cfg["T"],
         "recompute": "%d/%d tokens per row" % (n, cfg["T"]),
-        "schedule": "full for k<%d and every %d steps; cond cache reused every other cached step" % (
-            cfg["k0"], cfg["tau"]),
+        "schedule": "full for k<%d and every %d steps; %s" % (
+            cfg["k0"], cfg["tau"], "no condition cache" if cfg["tau_cfg"] == 0 else
+            "cond cache reused on cached steps with (k-k0) %% %d != 0" % cfg["tau_cfg"]),
         "decoding_steps": cfg["steps"],
-        "l2": "no flush: the per-step working set (0.34 GB weights + 1.3 GB K/V cache) exceeds the 129 MB L2",
+        "l2": "no flush: the per-step working set (%.2f GB weights + %.2f GB K/V cache) exceeds the 129 MB L2" % (
+            12 * cfg["depth"] * cfg["width"] ** 2 * 2 / 1e9,
+            2 * (cfg["depth"] - cfg["sel_layers"]) * 2 * cfg["batch"] * cfg["T"] * cfg["width"] * 2 / 1e9),
     }
 
 
@@ -382,9 +390,12 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", default="mar_b")
+    ap.add_argument("--ratio", type=float, default=None, help="recompute ratio (default: the config's)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     cfg = synth.config(args.config)
+    if args.ratio is not None:
+        cfg["ratio"] = args.ratio
     if args.impl == "reference":
         import oracle as O
         plan = [O.plan(k, cfg["k0"], cfg["tau"], cfg["tau_cfg"]) for k in range(cfg["steps"])]
