@@ -350,8 +350,8 @@ def run_ours(args, cfg):
                          "tflops": round(v["flops"] / (v["ms"] / 1e3) / 1e12, 2) if v["flops"] and v["ms"] else None,
                          "gbs": round(v["bytes"] / (v["ms"] / 1e3) / 1e9, 1) if v["ms"] else None}
     traffic = None
-    tpath = os.path.join(ROOT, "profiles", "gemm_traffic.json")
-    if os.path.exists(tpath):
+    tpath = os.path.join(ROOT, "profiles", "gemm_traffic.json")  # captured on the MAR-B decode
+    if cfg["name"] == "mar_b" and os.path.exists(tpath):
         with open(tpath) as f:
             traffic = json.load(f).get("bytes_per_launch")
     line = {
