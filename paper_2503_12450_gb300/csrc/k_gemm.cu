@@ -141,8 +141,13 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // Tiles are numbered column-tile fastest: the CTAs running at the same time
+  // cover a few row tiles completely, so each activation row tile is fetched
+  // from memory once and shared through L2 by the CTAs that use it (the
+  // weights, at most a few MB, stay in L2 throughout).
   const int num_m = (M + tc::BM - 1) / tc::BM;
-  const int tiles = num_m * (N / BN);
+  const int num_n = N / BN;
+  const int tiles = num_m * num_n;
   const int KB = K / tc::BK;
 
   if (threadIdx.x == 0) {
@@ -172,7 +177,7 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
   // every other access follows pdl_wait().
   int pre = 0;
   if (warp == 0 && lane == 0 && (int)blockIdx.x < tiles) {
-    const int n0 = ((int)blockIdx.x / num_m) * BN;
+    const int n0 = ((int)blockIdx.x % num_n) * BN;
     pre = KB < C::STAGES ? KB : C::STAGES;
     for (int s = 0; s < pre; ++s) {
       mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
@@ -189,7 +194,7 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
       uint32_t phase = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
-        const int m0 = (tile % num_m) * tc::BM, n0 = (tile / num_m) * BN;
+        const int m0 = (tile / num_n) * tc::BM, n0 = (tile % num_n) * BN;
         for (int kb = 0; kb < KB; ++kb) {
           if (tile == (int)blockIdx.x && kb < pre) {
             // weight tile already in flight on this stage: add the activations
@@ -255,7 +260,7 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++it) {
       const int buf = it & 1;
       const uint32_t use = (uint32_t)(it >> 1) & 1u;
-      const int m0 = (tile % num_m) * tc::BM, n0 = (tile / num_m) * BN;
+      const int m0 = (tile / num_n) * tc::BM, n0 = (tile % num_n) * BN;
       const int rbase = m0 + quarter * 32;  // first of this warp's 32 rows
       const int c0 = half * CHUNKS;
       // residual of a 32-column chunk in the coalesced layout: [16-col half][pass]
