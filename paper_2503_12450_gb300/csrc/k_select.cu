@@ -59,11 +59,149 @@ __global__ void __launch_bounds__(256) similarity_kernel(const T* __restrict__ c
   }
 }
 
+// bf16 similarity on the integer pipe (GB300's fp64 rate is a small fraction
+// of its integer rate). A bf16 value is M * 2^(E - 134) with an 8-bit integer
+// significand M (hidden bit included) and E = max(biased exponent, 1), so a
+// product of two is (Ma Mb) * 2^(Ea + Eb - 268) with Ma Mb < 2^16. Each sum
+// is taken relative to a base exponent kSpan = 62 - 16 - ceil(log2 D) below
+// its largest possible term exponent (from the vectors' largest exponents):
+// shifted to the base, every term is an integer below 2^(16 + kSpan) and the
+// D-term sum is exact in an int64. Its conversion to double is then the
+// correctly rounded exact sum, which equals the fp64 sum of the same products
+// whenever that sum is exact. A token with a nonzero term below the base, or
+// with an Inf/NaN element, takes the fp64 loop of similarity_kernel instead.
+// Each lane keeps its NCH 8-element chunks of both vectors in registers
+// (D <= 1280; wider vectors use similarity_kernel).
+template <int NCH>
+__global__ void __launch_bounds__(256) similarity_int_kernel(const bf16* __restrict__ cur, bf16* __restrict__ cache,
+                                                             double* __restrict__ S, long long ntok, int D, int span,
+                                                             int copy) {
+  pdl_wait();
+  pdl_trigger();
+  const long long tok = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (tok >= ntok) return;
+  const bf16* a = cur + tok * D;
+  bf16* c = cache + tok * D;
+  uint4 ra[NCH], rc[NCH];
+#pragma unroll
+  for (int j = 0; j < NCH; ++j) {
+    const int i = (lane + 32 * j) * 8;
+    if (i < D) {
+      ra[j] = *reinterpret_cast<const uint4*>(a + i);
+      rc[j] = *reinterpret_cast<const uint4*>(c + i);
+    } else {
+      ra[j] = make_uint4(0, 0, 0, 0);
+      rc[j] = make_uint4(0, 0, 0, 0);
+    }
+  }
+  // largest exponent field of each vector (two bf16 per 32-bit word)
+  uint32_t xa = 0, xc = 0;
+#pragma unroll
+  for (int j = 0; j < NCH; ++j) {
+    xa = __vmaxu2(xa, __vmaxu2(ra[j].x & 0x7F807F80u, ra[j].y & 0x7F807F80u));
+    xa = __vmaxu2(xa, __vmaxu2(ra[j].z & 0x7F807F80u, ra[j].w & 0x7F807F80u));
+    xc = __vmaxu2(xc, __vmaxu2(rc[j].x & 0x7F807F80u, rc[j].y & 0x7F807F80u));
+    xc = __vmaxu2(xc, __vmaxu2(rc[j].z & 0x7F807F80u, rc[j].w & 0x7F807F80u));
+  }
+  int ema = max((int)((xa >> 7) & 0xFFu), (int)((xa >> 23) & 0xFFu));
+  int emc = max((int)((xc >> 7) & 0xFFu), (int)((xc >> 23) & 0xFFu));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    ema = max(ema, __shfl_xor_sync(0xffffffffu, ema, o));
+    emc = max(emc, __shfl_xor_sync(0xffffffffu, emc, o));
+  }
+  bool inexact = ema == 255 || emc == 255;  // Inf or NaN present
+  ema = max(ema, 1);
+  emc = max(emc, 1);
+  const int bd = ema + emc - span, ba = 2 * ema - span, bc = 2 * emc - span;
+  long long sd = 0, sa = 0, sc = 0;
+  if (!inexact) {
+#pragma unroll
+    for (int j = 0; j < NCH; ++j) {
+      const uint32_t wa[4] = {ra[j].x, ra[j].y, ra[j].z, ra[j].w}, wc[4] = {rc[j].x, rc[j].y, rc[j].z, rc[j].w};
+#pragma unroll
+      for (int h = 0; h < 8; ++h) {
+        const uint32_t ya = (wa[h >> 1] >> (16 * (h & 1))) & 0xFFFFu, yc = (wc[h >> 1] >> (16 * (h & 1))) & 0xFFFFu;
+        const int ea = (int)((ya >> 7) & 0xFFu), ec = (int)((yc >> 7) & 0xFFu);
+        const int Ea = max(ea, 1), Ec = max(ec, 1);
+        const uint32_t Ma = (ya & 0x7Fu) | (ea ? 0x80u : 0u), Mc = (yc & 0x7Fu) | (ec ? 0x80u : 0u);
+        const uint32_t pd = Ma * Mc, pa = Ma * Ma, pc = Mc * Mc;
+        const int hd = Ea + Ec - bd, ha = 2 * Ea - ba, hc = 2 * Ec - bc;
+        inexact |= (hd < 0 && pd != 0) | (ha < 0 && pa != 0) | (hc < 0 && pc != 0);
+        const long long td = (long long)((unsigned long long)pd << max(hd, 0));
+        sd += ((ya ^ yc) & 0x8000u) ? -td : td;
+        sa += (long long)((unsigned long long)pa << max(ha, 0));
+        sc += (long long)((unsigned long long)pc << max(hc, 0));
+      }
+    }
+  }
+  double dot, na, nc;
+  if (__any_sync(0xffffffffu, inexact)) {
+    // fp64 fallback (the arithmetic of similarity_kernel)
+    dot = 0.0, na = 0.0, nc = 0.0;
+#pragma unroll 1
+    for (int i = lane * 8; i < D; i += 256) {
+      float av[8], cv[8];
+      Vec<bf16, 8>::load(a + i, av);
+      Vec<bf16, 8>::load(c + i, cv);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const double x = (double)av[k], y = (double)cv[k];
+        dot = fma(x, y, dot);
+        na = fma(x, x, na);
+        nc = fma(y, y, nc);
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      dot += __shfl_xor_sync(0xffffffffu, dot, o);
+      na += __shfl_xor_sync(0xffffffffu, na, o);
+      nc += __shfl_xor_sync(0xffffffffu, nc, o);
+    }
+  } else {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      sd += __shfl_xor_sync(0xffffffffu, sd, o);
+      sa += __shfl_xor_sync(0xffffffffu, sa, o);
+      sc += __shfl_xor_sync(0xffffffffu, sc, o);
+    }
+    dot = ldexp((double)sd, bd - 268);
+    na = ldexp((double)sa, ba - 268);
+    nc = ldexp((double)sc, bc - 268);
+  }
+  if (copy) {
+#pragma unroll
+    for (int j = 0; j < NCH; ++j) {
+      const int i = (lane + 32 * j) * 8;
+      if (i < D) *reinterpret_cast<uint4*>(c + i) = ra[j];
+    }
+  }
+  if (lane == 0) {
+    const double eps = 1e-8;
+    S[tok] = dot / sqrt(fmax(na * nc, eps * eps));
+  }
+}
+
 cudaError_t launch_similarity(const Ctx& c, int dtype, const void* cur, void* cache, double* S, int rows, int T, int D,
                               bool copy) {
   const long long ntok = (long long)rows * T;
   if (ntok == 0) return cudaSuccess;
   const unsigned grid = (unsigned)((ntok + 7) / 8);
+  if (dtype == LAZYMAR_BF16 && D % 8 == 0 && D <= 1280) {
+    int lg = 0;
+    while ((1 << lg) < D) ++lg;
+    const int span = 62 - 16 - lg;
+    const int nch = (D + 255) / 256;
+    const bf16* a = static_cast<const bf16*>(cur);
+    bf16* k = static_cast<bf16*>(cache);
+    const int cp = copy ? 1 : 0;
+    if (nch <= 1) return launch_pdl(similarity_int_kernel<1>, dim3(grid), dim3(256), 0, c.stream, a, k, S, ntok, D, span, cp);
+    if (nch <= 2) return launch_pdl(similarity_int_kernel<2>, dim3(grid), dim3(256), 0, c.stream, a, k, S, ntok, D, span, cp);
+    if (nch <= 3) return launch_pdl(similarity_int_kernel<3>, dim3(grid), dim3(256), 0, c.stream, a, k, S, ntok, D, span, cp);
+    if (nch <= 4) return launch_pdl(similarity_int_kernel<4>, dim3(grid), dim3(256), 0, c.stream, a, k, S, ntok, D, span, cp);
+    return launch_pdl(similarity_int_kernel<5>, dim3(grid), dim3(256), 0, c.stream, a, k, S, ntok, D, span, cp);
+  }
   if (dtype == LAZYMAR_BF16)
     return launch_pdl(similarity_kernel<bf16>, dim3(grid), dim3(256), 0, c.stream, (const bf16*)cur, (bf16*)cache, S,
                       ntok, D, copy ? 1 : 0);

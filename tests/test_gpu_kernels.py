@@ -42,6 +42,62 @@ def test_select_tokens_bit_exact(rows, T, D, N, dtype):
     assert torch.equal(g_ref, g_cur)
 
 
+def _selection_edge_inputs(T, D, seed):
+    """bf16 rows that exercise both similarity paths of the kernel.
+
+    row 0: every element scaled by 2^u, u uniform in [-60, 60] (exponent span
+           far beyond the exact integer sums: the fp64 path);
+    row 1: per token either a narrow ([-4, 4]) or a wide ([-30, 30]) span;
+    row 2: subnormal and near-subnormal values, zero tokens, cur = -ref;
+    row 3: Inf / NaN elements in a few tokens (S is NaN, ranked as -inf).
+    """
+    rng = np.random.Generator(np.random.PCG64(seed))
+    ref = rng.standard_normal((4, T, D)).astype(np.float32)
+    cur = ref * (1 + 0.05 * rng.standard_normal((4, T, D))).astype(np.float32)
+    big = rng.random((4, T)) < 0.2
+    cur[big] = rng.standard_normal((int(big.sum()), D)).astype(np.float32)
+    u = rng.integers(-60, 61, size=(T, D))
+    cur[0] *= np.exp2(u).astype(np.float32)
+    ref[0] *= np.exp2(u).astype(np.float32)
+    span = np.where(rng.random(T) < 0.5, 4, 30)[:, None]
+    u = rng.integers(-span, span + 1, size=(T, D))
+    cur[1] *= np.exp2(u).astype(np.float32)
+    ref[1] *= np.exp2(u).astype(np.float32)
+    scale = np.where(rng.random((T, 1)) < 0.5, 2.0 ** -130, 2.0 ** -120).astype(np.float32)
+    cur[2] *= scale
+    ref[2] *= scale
+    cur[2, :5] = 0.0
+    ref[2, 3:8] = 0.0
+    cur[2, 10:20] = -ref[2, 10:20]
+    for t, v in [(0, np.inf), (7, -np.inf), (11, np.nan)]:
+        cur[3, t, t % D] = v
+    ref[3, 20, 5] = np.inf
+    ref[3, 21, 6] = np.nan
+    return synth.round_bf16(cur), synth.round_bf16(ref)
+
+
+@pytest.mark.parametrize("D", [768, 1280, 64])
+def test_select_tokens_exponent_range_and_specials(D):
+    """Selections agree with the oracle on data whose exponent spans, subnormals
+    and Inf/NaN elements steer tokens through both the exact integer sums and
+    the fp64 fallback. (Where the spans exceed what fp64 sums exactly, both
+    sides round; the random data has no near-ties for that to reorder.)"""
+    torch = torch_cuda()
+    T, N = 200, 60
+    cur, ref = _selection_edge_inputs(T, D, seed=D)
+    g_cur, g_ref = dev(cur, "bf16"), dev(ref, "bf16")
+    idx = torch.full((4, N), -1, dtype=torch.int32, device="cuda")
+    lm.lazymar_select_tokens(DT["bf16"], g_cur, g_ref, 4, T, D, N, idx)
+    sync()
+    got = idx.cpu().numpy()
+    with np.errstate(invalid="ignore", over="ignore"):
+        for r in range(4):
+            expect = O.select_compute(O.cosine_similarity(cur[r], ref[r]), N)
+            assert got[r].tolist() == expect.tolist(), "row %d" % r
+    # bit patterns: the copied NaNs compare unequal as values
+    assert torch.equal(g_ref.view(torch.int16), g_cur.view(torch.int16))
+
+
 # --------------------------------------------------------------------------
 # Condition cache / guidance (Eq. 7 reading, Eq. 10)
 # --------------------------------------------------------------------------
