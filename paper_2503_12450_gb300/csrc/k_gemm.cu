@@ -83,11 +83,14 @@ enum EpiKind { BF16OUT = 0, RESID_WIDE = 1, RESID_HALF = 2 };
 
 template <int BN, int EK>
 struct Cfg {
-  static constexpr int STAGES = EK == RESID_WIDE ? (BN == 256 ? 3 : 5) : (BN == 256 ? 4 : 6);
+  static constexpr int STAGES = EK == RESID_WIDE ? (BN == 256 ? 3 : BN == 192 ? 4 : 5)
+                                                  : (BN == 256 ? 4 : BN == 192 ? 5 : 6);
   static constexpr uint32_t A_BYTES = BM * BK * 2;
   static constexpr uint32_t B_BYTES = BN * BK * 2;
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulator buffers
+  // two accumulator buffers (columns [0, BN) and [BN, 2 BN)); the allocation
+  // is a power of two
+  static constexpr uint32_t TMEM_COLS = 2 * BN <= 256 ? 256 : 512;
   // Per-warp staging of 32 rows (64 or 128 bytes each), rows padded by 16
   // bytes so that both the row-wise writes and the column-block reads are
   // bank-conflict-lean.
@@ -534,20 +537,35 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
     return launch_pdl(gemm_f32_kernel, grid, dim3(256), 0, c.stream, static_cast<const float*>(A),
                       static_cast<const float*>(W), M, N, K, epi);
   }
-  // Tile width: the one with fewer tile-waves x tile-time over the SMs.
+  // Tile width: the one with the fewest rounds of tiles over the SMs x the
+  // time of one tile. Relative tile times 225 : 243 : 256 for BN = 128 : 192 :
+  // 256 (measured, one round of 128 x BN x 3072 tiles): narrower tiles are
+  // capped by shared-memory operand bandwidth well below the BN = 256 rate.
   int bn = 128;
   if (flags == 2 && N % 256 == 0) {
     bn = 256;
-  } else if (flags == 0 && N % 256 == 0) {
+  } else if (flags == 3 && N % 192 == 0) {
+    bn = 192;
+  } else if (flags == 0) {
     const long mt = (M + tc::BM - 1) / tc::BM;
-    const long w128 = (mt * (N / 128) + c.num_sms - 1) / c.num_sms;  // waves of BN = 128 tiles
-    const long w256 = (mt * (N / 256) + c.num_sms - 1) / c.num_sms;  // waves of BN = 256 tiles
-    // A BN = 128 tile is capped by shared-memory bandwidth at about 0.56x the
-    // main-loop rate of a BN = 256 tile (measured), so BN = 256 wins unless it
-    // leaves more than 1.12x as many tile-waves idle.
-    if (w256 * 112 <= w128 * 100) bn = 256;
+    long best = -1;
+    const int widths[3] = {256, 192, 128}, tile_time[3] = {256, 243, 225};
+    for (int i = 0; i < 3; ++i) {
+      if (N % widths[i] != 0) continue;
+      const long rounds = (mt * (N / widths[i]) + c.num_sms - 1) / c.num_sms;
+      const long cost = rounds * tile_time[i];
+      if (best < 0 || cost < best) {
+        best = cost;
+        bn = widths[i];
+      }
+    }
   }
   const int ek = epi.mode != LAZYMAR_EPI_RESIDUAL ? tc::BF16OUT : (K < 2048 ? tc::RESID_WIDE : tc::RESID_HALF);
+  if (bn == 192) {
+    if (ek == tc::RESID_WIDE) return launch_tc<192, tc::RESID_WIDE>(c, A, W, M, N, K, epi);
+    if (ek == tc::RESID_HALF) return launch_tc<192, tc::RESID_HALF>(c, A, W, M, N, K, epi);
+    return launch_tc<192, tc::BF16OUT>(c, A, W, M, N, K, epi);
+  }
   if (bn == 256) {
     if (ek == tc::RESID_WIDE) return launch_tc<256, tc::RESID_WIDE>(c, A, W, M, N, K, epi);
     if (ek == tc::RESID_HALF) return launch_tc<256, tc::RESID_HALF>(c, A, W, M, N, K, epi);
