@@ -383,6 +383,48 @@ def run_ours(args, cfg):
         dist.destroy_process_group()
 
 
+def profile_case(args, cfg):
+    """One launch of each kernel of a layer at the configuration's shapes, for a
+    profiler: `gemm_layers` runs QKV, out-proj, fc1 and fc2 on all rows x T
+    tokens and on the recomputed rows x N tokens; `attention_layers` runs the
+    recomputed-token and the full-layer attention."""
+    import torch
+    from paper_2503_12450_gb300 import lazymar as lm
+    lm.lib()
+    torch.manual_seed(0)
+    rows, T, D, H = 2 * cfg["batch"], cfg["T"], cfg["width"], cfg["heads"]
+    N = synth.n_compute(cfg)
+    dev = "cuda"
+    if args.profile_case == "gemm_layers":
+        for M in (rows * T, rows * N):
+            for n, k, epi in [(3 * D, D, lm.LAZYMAR_EPI_QKV), (D, D, lm.LAZYMAR_EPI_RESIDUAL),
+                              (4 * D, D, lm.LAZYMAR_EPI_GELU), (D, 4 * D, lm.LAZYMAR_EPI_RESIDUAL)]:
+                a = torch.randn(M, k, device=dev).bfloat16()
+                w = (torch.randn(n, k, device=dev) * 0.05).bfloat16()
+                b = torch.randn(n, device=dev).bfloat16()
+                if epi == lm.LAZYMAR_EPI_QKV:
+                    q = torch.empty(M, D, device=dev, dtype=torch.bfloat16)
+                    kk, vv = torch.empty_like(q), torch.empty_like(q)
+                    lm.lazymar_linear(lm.LAZYMAR_BF16, epi, a, w, b, M, n, k, q, D, kk, vv, None)
+                elif epi == lm.LAZYMAR_EPI_RESIDUAL:
+                    o = torch.zeros(M, n, device=dev)
+                    lm.lazymar_linear(lm.LAZYMAR_BF16, epi, a, w, b, M, n, k, o, n)
+                else:
+                    o = torch.empty(M, n, device=dev, dtype=torch.bfloat16)
+                    lm.lazymar_linear(lm.LAZYMAR_BF16, epi, a, w, b, M, n, k, o, n)
+                torch.cuda.synchronize()
+    else:
+        for nq in (N, T):
+            q = torch.randn(rows * nq, D, device=dev).bfloat16()
+            k = torch.randn(rows * T, D, device=dev).bfloat16()
+            v = torch.randn_like(k)
+            o = torch.empty_like(q)
+            lm.lazymar_attention(lm.LAZYMAR_BF16, q, k, v, o, rows, nq, T, H, D // H)
+            torch.cuda.synchronize()
+    lm.lazymar_device_check()
+    print(json.dumps({"profile_case": args.profile_case, "config": cfg["name"], "ok": True}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -392,11 +434,15 @@ def main():
     ap.add_argument("--config", default="mar_b")
     ap.add_argument("--ratio", type=float, default=None, help="recompute ratio (default: the config's)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile-case", choices=["gemm_layers", "attention_layers"], default=None,
+                    help="run each kernel of a layer once at the configuration's shapes (for ncu) and exit")
     args = ap.parse_args()
     cfg = synth.config(args.config)
     if args.ratio is not None:
         cfg["ratio"] = args.ratio
-    if args.impl == "reference":
+    if args.profile_case:
+        profile_case(args, cfg)
+    elif args.impl == "reference":
         import oracle as O
         plan = [O.plan(k, cfg["k0"], cfg["tau"], cfg["tau_cfg"]) for k in range(cfg["steps"])]
         run_reference(args, cfg, plan)
