@@ -54,25 +54,30 @@ __device__ __forceinline__ float exp2_approx(float x) {
   return y;
 }
 
-// GELU(x) = x * Phi(x) = 0.5 x (1 + erf(x / sqrt 2)), with erf from the
-// rational approximation of Abramowitz & Stegun, Handbook of Mathematical
-// Functions, formula 7.1.26: for z >= 0,
-//   erf(z) = 1 - (a1 t + a2 t^2 + a3 t^3 + a4 t^4 + a5 t^5) exp(-z^2),
-//   t = 1 / (1 + p z),  |error| <= 1.5e-7,
-// and erf(-z) = -erf(z). Branch-free, two special-function instructions and a
-// handful of FMAs per element: the MLP epilogue applies it to every element of
-// the 4D-wide hidden layer and is instruction-bound.
+// GELU(x) = x Phi(x) = max(x, 0) - |x| h(|x|), where h(u) = Phi(-u) =
+// erfc(u / sqrt 2) / 2 is the normal tail. h is evaluated as 2^P(u) with P a
+// degree-5 polynomial fitted to log2 h on u in [0, 6] (weighted least squares
+// towards minimax; coefficients from csrc/gen_gelu_poly.py); u is clamped to 6,
+// where h < 1e-9. In fp32 the result is within 2.8e-7 * max(1, |x|) of the
+// exact erf GELU. Per element: one special-function instruction and eight
+// ALU ones (the MLP epilogue applies it to every element of the 4D-wide
+// hidden layer and is instruction-bound). The ReLU term is (x + |x|) / 2 so
+// that a NaN input stays NaN.
 __device__ __forceinline__ float gelu_erf(float x) {
-  const float z = fabsf(x) * 0.70710678118654752f;
-  const float t = rcp_approx(fmaf(0.3275911f, z, 1.0f));
-  float poly = fmaf(1.061405429f, t, -1.453152027f);
-  poly = fmaf(poly, t, 1.421413741f);
-  poly = fmaf(poly, t, -0.284496736f);
-  poly = fmaf(poly, t, 0.254829592f);
-  poly *= t;
-  const float e = exp2_approx(-z * z * 1.4426950408889634f);
-  const float erf_abs = fmaf(-poly, e, 1.0f);
-  return 0.5f * x * (1.0f + copysignf(erf_abs, x));
+  constexpr float kGeluP0 = -1.000018716e+00f;
+  constexpr float kGeluP1 = -1.150941610e+00f;
+  constexpr float kGeluP2 = -4.596132934e-01f;
+  constexpr float kGeluP3 = -5.220982432e-02f;
+  constexpr float kGeluP4 = 7.249599788e-03f;
+  constexpr float kGeluP5 = -4.984181724e-04f;
+  const float u = fminf(fabsf(x), 6.0f);
+  float p = fmaf(kGeluP5, u, kGeluP4);
+  p = fmaf(p, u, kGeluP3);
+  p = fmaf(p, u, kGeluP2);
+  p = fmaf(p, u, kGeluP1);
+  p = fmaf(p, u, kGeluP0);
+  const float h = exp2_approx(p);
+  return fmaf(-u, h, 0.5f * (x + fabsf(x)));
 }
 
 __device__ __forceinline__ float warp_sum(float v) {
