@@ -71,8 +71,6 @@ __device__ __forceinline__ void epilogue_apply(const GemmEpi& e, int row, int co
 namespace tc {
 constexpr int BM = 128;  // rows per tile = MMA M (one accumulator lane per row)
 constexpr int BK = 64;   // one 128-byte swizzle atom of bf16 along K
-constexpr int kEpiWarps = 8;
-constexpr int kThreads = 64 + kEpiWarps * 32;
 
 // Epilogue kinds: BF16OUT stores bf16 (bias / GELU / Q-K-V split); the two
 // residual kinds add into the fp32 residual stream. RESID_WIDE stages whole
@@ -94,10 +92,19 @@ struct Cfg {
   // Per-warp staging of 32 rows (64 or 128 bytes each), rows padded by 16
   // bytes so that both the row-wise writes and the column-block reads are
   // bank-conflict-lean.
+  // Epilogue warps: the bf16-output kinds use four (three for BN = 192) per
+  // tensor-memory lane quarter, so more warps share a tile's conversion,
+  // GELU and stores; the residual kinds, with more live registers, two.
+  static constexpr int EPI_WARPS = EK != BF16OUT ? 8 : (BN == 192 ? 12 : 16);
+  static constexpr int THREADS = 64 + EPI_WARPS * 32;
+  static constexpr int CHUNKS = BN / 32 / (EPI_WARPS / 4);  // 32-column chunks per warp and tile
+  // Per-warp staging of 32 rows: bf16 rows of 64 bytes, 16-byte blocks
+  // swizzled by row (conflict-free row-wise writes and column-block reads);
+  // fp32 rows of 64 or 128 bytes padded by 16 bytes.
   static constexpr uint32_t ROW_BYTES = EK == RESID_WIDE ? 128 : 64;
-  static constexpr uint32_t STG_PITCH = ROW_BYTES + 16;
+  static constexpr uint32_t STG_PITCH = EK == BF16OUT ? 64 : ROW_BYTES + 16;
   static constexpr uint32_t STG_BYTES = 32 * STG_PITCH;
-  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + kEpiWarps * STG_BYTES + 256;
+  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + EPI_WARPS * STG_BYTES + 256;
   // Instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1),
   // B bf16 (bits 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
   static constexpr uint32_t IDESC =
@@ -126,7 +133,7 @@ __device__ __forceinline__ bf16* out_row(const GemmEpi& e, int row, int col) {
 }  // namespace tc
 
 template <int BN, int EK>
-__global__ void __launch_bounds__(tc::kThreads, 1)
+__global__ void __launch_bounds__(tc::Cfg<BN, EK>::THREADS, 1)
     gemm_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M,
                         int N, int K, GemmEpi epi, unsigned* err) {
   using C = tc::Cfg<BN, EK>;
@@ -136,7 +143,7 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
   uint8_t* sA = smem;
   uint8_t* sB = smem + C::STAGES * C::A_BYTES;
   uint8_t* sStg = smem + C::STAGES * C::STAGE_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sStg + tc::kEpiWarps * C::STG_BYTES);
+  uint64_t* full = reinterpret_cast<uint64_t*>(sStg + C::EPI_WARPS * C::STG_BYTES);
   uint64_t* empty = full + C::STAGES;
   uint64_t* acc_full = empty + C::STAGES;
   uint64_t* acc_empty = acc_full + 2;
@@ -160,7 +167,7 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
-      mbar_init(&acc_empty[b], tc::kEpiWarps);
+      mbar_init(&acc_empty[b], C::EPI_WARPS);
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -243,18 +250,19 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
     __syncwarp();
   } else {
     // ---------------- epilogue warps ----------------
-    // Each warp owns 32 accumulator rows (its TMEM lane quarter) and half of
-    // the tile's columns, processed as 32 x 32 chunks. tcgen05.ld gives one row
+    // Each warp owns 32 accumulator rows (its TMEM lane quarter) and one of the
+    // EPI_WARPS / 4 column ranges of the tile, processed as 32 x 32 chunks
+    // (CHUNKS per tile). tcgen05.ld gives one row
     // per thread; each chunk is transposed through the warp's staging buffer
     // (32 rows x 64 bytes: 32 bf16 columns, or 16 fp32 columns at a time) so
     // that every global store and residual load covers 8 rows x 64 contiguous
     // bytes per warp instruction. The residual of the next chunk is loaded
     // while the current one is processed, and the first chunk's before the
     // accumulator is ready.
-    const int ew = warp - 2;        // 0..7
+    const int ew = warp - 2;        // 0 .. EPI_WARPS - 1
     const int quarter = warp & 3;   // tensor-memory lanes this warp may read
-    const int half = ew >> 2;       // which half of the tile's columns
-    constexpr int CHUNKS = BN / 64; // 32-column chunks per half
+    const int half = ew >> 2;       // which column range of the tile (of EPI_WARPS / 4)
+    constexpr int CHUNKS = C::CHUNKS;
     uint8_t* stg = sStg + ew * C::STG_BYTES;
     const int cr = lane >> 2;       // row within an 8-row pass
     const int cq = lane & 3;        // 16-byte block within the 64-byte row segment
@@ -386,13 +394,22 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = gelu_erf(v[i]);
           }
-          Vec<bf16, 32>::store(reinterpret_cast<bf16*>(stg + lane * C::STG_PITCH), v);
+          {
+            // row `lane`, 16-byte block j at block j ^ ((lane >> 1) & 3)
+            uint4 pk[4];
+            uint32_t* w = reinterpret_cast<uint32_t*>(pk);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) w[i] = pack_bf16(v[2 * i], v[2 * i + 1]);
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              *reinterpret_cast<uint4*>(stg + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4)) = pk[j];
+          }
           __syncwarp();
 #pragma unroll
           for (int p = 0; p < 4; ++p) {
             const int lr = p * 8 + cr;
             const int row = rbase + lr;
-            const uint4 val = *reinterpret_cast<const uint4*>(stg + lr * C::STG_PITCH + cq * 16);
+            const uint4 val = *reinterpret_cast<const uint4*>(stg + lr * 64 + ((cq ^ ((lr >> 1) & 3)) << 4));
             if (row < M) *reinterpret_cast<uint4*>(tc::out_row(epi, row, col) + cq * 8) = val;
           }
           __syncwarp();
@@ -525,7 +542,7 @@ static cudaError_t launch_tc(const Ctx& c, const void* A, const void* W, int M, 
   }
   const int tiles = ((M + tc::BM - 1) / tc::BM) * (N / BN);
   const int grid = tiles < c.num_sms ? tiles : c.num_sms;
-  return launch_pdl(gemm_bf16_tc_kernel<BN, EK>, dim3(grid), dim3(tc::kThreads), C::SMEM, c.stream, ta, tb, M, N, K,
+  return launch_pdl(gemm_bf16_tc_kernel<BN, EK>, dim3(grid), dim3(C::THREADS), C::SMEM, c.stream, ta, tb, M, N, K,
                     epi, c.err);
 }
 
