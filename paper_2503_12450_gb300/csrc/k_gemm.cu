@@ -16,6 +16,8 @@
 
 #include <mutex>
 
+#include <cstring>
+
 #include "lazymar_internal.cuh"
 
 namespace lm {
@@ -134,8 +136,10 @@ __device__ __forceinline__ bf16* out_row(const GemmEpi& e, int row, int col) {
 
 template <int BN, int EK>
 __global__ void __launch_bounds__(tc::Cfg<BN, EK>::THREADS, 1)
-    gemm_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M,
-                        int N, int K, GemmEpi epi, unsigned* err) {
+    gemm_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                        const __grid_constant__ CUtensorMap tmO0, const __grid_constant__ CUtensorMap tmO1,
+                        const __grid_constant__ CUtensorMap tmO2, int tma_out, int M, int N, int K, GemmEpi epi,
+                        unsigned* err) {
   using C = tc::Cfg<BN, EK>;
   constexpr bool RESID = EK != tc::BF16OUT;
   extern __shared__ uint8_t smem_raw[];
@@ -394,31 +398,50 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK>::THREADS, 1)
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = gelu_erf(v[i]);
           }
+          uint4 pk[4];
           {
-            // row `lane`, 16-byte block j at block j ^ ((lane >> 1) & 3)
-            uint4 pk[4];
             uint32_t* w = reinterpret_cast<uint32_t*>(pk);
 #pragma unroll
             for (int i = 0; i < 16; ++i) w[i] = pack_bf16(v[2 * i], v[2 * i + 1]);
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-              *reinterpret_cast<uint4*>(stg + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4)) = pk[j];
           }
-          __syncwarp();
-#pragma unroll
-          for (int p = 0; p < 4; ++p) {
-            const int lr = p * 8 + cr;
-            const int row = rbase + lr;
-            const uint4 val = *reinterpret_cast<const uint4*>(stg + lr * 64 + ((cq ^ ((lr >> 1) & 3)) << 4));
-            if (row < M) *reinterpret_cast<uint4*>(tc::out_row(epi, row, col) + cq * 8) = val;
+          if (tma_out) {
+            // the previous chunk's store must have read the staging buffer
+            if (lane == 0) bulk_wait_read();
+            __syncwarp();
           }
-          __syncwarp();
+          // row `lane`, 16-byte block j at block j ^ ((lane >> 1) & 3): the
+          // TMA 64-byte swizzle of a 32 x 32 bf16 box
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            *reinterpret_cast<uint4*>(stg + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4)) = pk[j];
+          if (tma_out) {
+            // one TMA store of the 32 x 32 chunk; rows beyond M are clipped
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0 && rbase < M) {
+              const int part = epi.mode == LAZYMAR_EPI_QKV ? col / epi.D : 0;
+              const CUtensorMap* tm = part == 0 ? &tmO0 : part == 1 ? &tmO1 : &tmO2;
+              tma_store_2d(tm, stg, col - part * epi.D, rbase);
+              bulk_commit();
+            }
+          } else {
+            __syncwarp();
+#pragma unroll
+            for (int p = 0; p < 4; ++p) {
+              const int lr = p * 8 + cr;
+              const int row = rbase + lr;
+              const uint4 val = *reinterpret_cast<const uint4*>(stg + lr * 64 + ((cq ^ ((lr >> 1) & 3)) << 4));
+              if (row < M) *reinterpret_cast<uint4*>(tc::out_row(epi, row, col) + cq * 8) = val;
+            }
+            __syncwarp();
+          }
         }
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&acc_empty[buf]);
     }
+    if (tma_out && lane == 0) bulk_wait_all();  // stores complete before the CTA exits
   }
   __syncthreads();
   if (warp == 1) {
@@ -540,9 +563,28 @@ static cudaError_t launch_tc(const Ctx& c, const void* A, const void* W, int M, 
     if (e != cudaSuccess) return e;
     attr_set[dev] = 1;
   }
+  // bf16 outputs leave through TMA stores of 32 x 32 boxes (64-byte swizzle),
+  // except Q/K/V with a row map, whose K/V rows are scattered
+  CUtensorMap to[3];
+  std::memset(to, 0, sizeof to);
+  int tma_out = 0;
+  if (EK == tc::BF16OUT && !(epi.mode == LAZYMAR_EPI_QKV && epi.row_map)) {
+    tma_out = 1;
+    if (epi.mode == LAZYMAR_EPI_QKV) {
+      const void* outs[3] = {epi.out, epi.k_out, epi.v_out};
+      for (int i = 0; i < 3; ++i)
+        if (!make_tmap_bf16(&to[i], outs[i], (uint64_t)epi.D, (uint64_t)M, (uint64_t)epi.D * 2, 32, 32,
+                            CU_TENSOR_MAP_SWIZZLE_64B))
+          return cudaErrorInvalidValue;
+    } else if (!make_tmap_bf16(&to[0], epi.out, (uint64_t)N, (uint64_t)M, (uint64_t)epi.ldo * 2, 32, 32,
+                               CU_TENSOR_MAP_SWIZZLE_64B)) {
+      return cudaErrorInvalidValue;
+    }
+  }
   const int tiles = ((M + tc::BM - 1) / tc::BM) * (N / BN);
   const int grid = tiles < c.num_sms ? tiles : c.num_sms;
-  return launch_pdl(gemm_bf16_tc_kernel<BN, EK>, dim3(grid), dim3(C::THREADS), C::SMEM, c.stream, ta, tb, M, N, K,
+  return launch_pdl(gemm_bf16_tc_kernel<BN, EK>, dim3(grid), dim3(C::THREADS), C::SMEM, c.stream, ta, tb, to[0], to[1],
+                    to[2], tma_out, M, N, K,
                     epi, c.err);
 }
 
