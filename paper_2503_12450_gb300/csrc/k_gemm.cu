@@ -72,7 +72,7 @@ __device__ __forceinline__ void epilogue_apply(const GemmEpi& e, int row, int co
 // ---------------------------------------------------------------------------
 namespace tc {
 constexpr int BM = 128;  // rows per tile = MMA M (one accumulator lane per row)
-constexpr int BK = 64;   // one 128-byte swizzle atom of bf16 along K
+constexpr int ATOM_K = 64;  // one 128-byte swizzle atom of bf16 along K (one TMA box)
 
 // Epilogue kinds: BF16OUT stores bf16 (bias / GELU / Q-K-V split); the two
 // residual kinds add into the fp32 residual stream. RESID_WIDE stages whole
@@ -81,10 +81,16 @@ constexpr int BK = 64;   // one 128-byte swizzle atom of bf16 along K
 // every stage (for long K, where the main loop bounds it).
 enum EpiKind { BF16OUT = 0, RESID_WIDE = 1, RESID_HALF = 2 };
 
-template <int BN, int EK>
+// BK: K per pipeline stage, one or two swizzle atoms. A 128-wide tile runs
+// 128-deep stages (two atoms, eight MMAs per barrier round trip): its
+// 128 x 128 x 16 MMAs are too short to hide the per-stage wait and commit at
+// 64 (measured 13-19 % faster); wider tiles keep 64 for a deeper ring.
+template <int BN, int EK, int BK>
 struct Cfg {
-  static constexpr int STAGES = EK == RESID_WIDE ? (BN == 256 ? 3 : BN == 192 ? 4 : 5)
-                                                  : (BN == 256 ? 4 : BN == 192 ? 5 : 6);
+  static constexpr int ATOMS = BK / ATOM_K;
+  static constexpr int STAGES = BK == 128 ? (EK == RESID_WIDE ? 2 : 3)
+                                          : EK == RESID_WIDE ? (BN == 256 ? 3 : BN == 192 ? 4 : 5)
+                                                             : (BN == 256 ? 4 : BN == 192 ? 5 : 6);
   static constexpr uint32_t A_BYTES = BM * BK * 2;
   static constexpr uint32_t B_BYTES = BN * BK * 2;
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
@@ -134,13 +140,13 @@ __device__ __forceinline__ bf16* out_row(const GemmEpi& e, int row, int col) {
 }
 }  // namespace tc
 
-template <int BN, int EK>
-__global__ void __launch_bounds__(tc::Cfg<BN, EK>::THREADS, 1)
+template <int BN, int EK, int BK>
+__global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
     gemm_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                         const __grid_constant__ CUtensorMap tmO0, const __grid_constant__ CUtensorMap tmO1,
                         const __grid_constant__ CUtensorMap tmO2, int tma_out, int M, int N, int K, GemmEpi epi,
                         unsigned* err) {
-  using C = tc::Cfg<BN, EK>;
+  using C = tc::Cfg<BN, EK, BK>;
   constexpr bool RESID = EK != tc::BF16OUT;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -162,7 +168,7 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK>::THREADS, 1)
   const int num_m = (M + tc::BM - 1) / tc::BM;
   const int num_n = N / BN;
   const int tiles = num_m * num_n;
-  const int KB = K / tc::BK;
+  const int KB = K / BK;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
@@ -195,7 +201,9 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK>::THREADS, 1)
     pre = KB < C::STAGES ? KB : C::STAGES;
     for (int s = 0; s < pre; ++s) {
       mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
-      tma_load_2d(&tmB, &full[s], sB + s * C::B_BYTES, s * tc::BK, n0);
+#pragma unroll
+      for (int a = 0; a < C::ATOMS; ++a)
+        tma_load_2d(&tmB, &full[s], sB + s * C::B_BYTES + a * (C::B_BYTES / C::ATOMS), s * BK + a * tc::ATOM_K, n0);
     }
   }
   pdl_wait();
@@ -212,12 +220,20 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK>::THREADS, 1)
         for (int kb = 0; kb < KB; ++kb) {
           if (tile == (int)blockIdx.x && kb < pre) {
             // weight tile already in flight on this stage: add the activations
-            tma_load_2d(&tmA, &full[stage], sA + stage * C::A_BYTES, kb * tc::BK, m0);
+#pragma unroll
+            for (int a = 0; a < C::ATOMS; ++a)
+              tma_load_2d(&tmA, &full[stage], sA + stage * C::A_BYTES + a * (C::A_BYTES / C::ATOMS),
+                          kb * BK + a * tc::ATOM_K, m0);
           } else {
             if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
             mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
-            tma_load_2d(&tmA, &full[stage], sA + stage * C::A_BYTES, kb * tc::BK, m0);
-            tma_load_2d(&tmB, &full[stage], sB + stage * C::B_BYTES, kb * tc::BK, n0);
+#pragma unroll
+            for (int a = 0; a < C::ATOMS; ++a) {
+              tma_load_2d(&tmA, &full[stage], sA + stage * C::A_BYTES + a * (C::A_BYTES / C::ATOMS),
+                          kb * BK + a * tc::ATOM_K, m0);
+              tma_load_2d(&tmB, &full[stage], sB + stage * C::B_BYTES + a * (C::B_BYTES / C::ATOMS),
+                          kb * BK + a * tc::ATOM_K, n0);
+            }
           }
           if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
         }
@@ -243,8 +259,12 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK>::THREADS, 1)
           const uint64_t a0 = tc::sw128_desc(smem_u32(sA + stage * C::A_BYTES));
           const uint64_t b0 = tc::sw128_desc(smem_u32(sB + stage * C::B_BYTES));
 #pragma unroll
-          for (int k = 0; k < tc::BK / 16; ++k)  // +32 bytes per K=16 step inside the swizzle atom
-            umma_bf16(d_tmem, a0 + 2 * k, b0 + 2 * k, C::IDESC, (kb | k) != 0 ? 1u : 0u);
+          for (int k = 0; k < BK / 16; ++k) {  // +32 bytes per K=16 step inside an atom
+            const int a = k / (tc::ATOM_K / 16), ks = k % (tc::ATOM_K / 16);
+            const uint64_t ao = (uint64_t)((a * (C::A_BYTES / C::ATOMS)) >> 4) + 2 * ks;
+            const uint64_t bo = (uint64_t)((a * (C::B_BYTES / C::ATOMS)) >> 4) + 2 * ks;
+            umma_bf16(d_tmem, a0 + ao, b0 + bo, C::IDESC, (kb | k) != 0 ? 1u : 0u);
+          }
           umma_commit(&empty[stage]);
           if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
         }
@@ -546,19 +566,19 @@ bool gemm_supported(int dtype, int M, int N, int K, const GemmEpi& epi, const ch
   return true;
 }
 
-template <int BN, int EK>
+template <int BN, int EK, int BK>
 static cudaError_t launch_tc(const Ctx& c, const void* A, const void* W, int M, int N, int K, const GemmEpi& epi) {
-  using C = tc::Cfg<BN, EK>;
+  using C = tc::Cfg<BN, EK, BK>;
   CUtensorMap ta, tb;
-  if (!make_tmap_bf16(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * 2, tc::BK, tc::BM,
+  if (!make_tmap_bf16(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * 2, tc::ATOM_K, tc::BM,
                       CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !make_tmap_bf16(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, tc::BK, BN, CU_TENSOR_MAP_SWIZZLE_128B))
+      !make_tmap_bf16(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, tc::ATOM_K, BN, CU_TENSOR_MAP_SWIZZLE_128B))
     return cudaErrorInvalidValue;
   static int attr_set[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc_kernel<BN, EK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc_kernel<BN, EK, BK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)C::SMEM);
     if (e != cudaSuccess) return e;
     attr_set[dev] = 1;
@@ -583,7 +603,7 @@ static cudaError_t launch_tc(const Ctx& c, const void* A, const void* W, int M, 
   }
   const int tiles = ((M + tc::BM - 1) / tc::BM) * (N / BN);
   const int grid = tiles < c.num_sms ? tiles : c.num_sms;
-  return launch_pdl(gemm_bf16_tc_kernel<BN, EK>, dim3(grid), dim3(C::THREADS), C::SMEM, c.stream, ta, tb, to[0], to[1],
+  return launch_pdl(gemm_bf16_tc_kernel<BN, EK, BK>, dim3(grid), dim3(C::THREADS), C::SMEM, c.stream, ta, tb, to[0], to[1],
                     to[2], tma_out, M, N, K,
                     epi, c.err);
 }
@@ -597,9 +617,10 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
                       static_cast<const float*>(W), M, N, K, epi);
   }
   // Tile width: the one with the fewest rounds of tiles over the SMs x the
-  // time of one tile. Relative tile times 225 : 243 : 256 for BN = 128 : 192 :
-  // 256 (measured, one round of 128 x BN x 3072 tiles): narrower tiles are
-  // capped by shared-memory operand bandwidth well below the BN = 256 rate.
+  // time of one tile. Relative tile times 187 : 243 : 256 for BN = 128 : 192 :
+  // 256 (measured, one round of 128 x BN x 3072 tiles): a narrower tile does
+  // proportionally less work per pipeline stage and runs well below the
+  // BN = 256 rate.
   int bn = 128;
   if (flags == 2 && N % 256 == 0) {
     bn = 256;
@@ -608,7 +629,7 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
   } else if (flags == 0) {
     const long mt = (M + tc::BM - 1) / tc::BM;
     long best = -1;
-    const int widths[3] = {256, 192, 128}, tile_time[3] = {256, 243, 225};
+    const int widths[3] = {256, 192, 128}, tile_time[3] = {256, 243, 187};
     for (int i = 0; i < 3; ++i) {
       if (N % widths[i] != 0) continue;
       const long rounds = (mt * (N / widths[i]) + c.num_sms - 1) / c.num_sms;
@@ -621,18 +642,23 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
   }
   const int ek = epi.mode != LAZYMAR_EPI_RESIDUAL ? tc::BF16OUT : (K < 2048 ? tc::RESID_WIDE : tc::RESID_HALF);
   if (bn == 192) {
-    if (ek == tc::RESID_WIDE) return launch_tc<192, tc::RESID_WIDE>(c, A, W, M, N, K, epi);
-    if (ek == tc::RESID_HALF) return launch_tc<192, tc::RESID_HALF>(c, A, W, M, N, K, epi);
-    return launch_tc<192, tc::BF16OUT>(c, A, W, M, N, K, epi);
+    if (ek == tc::RESID_WIDE) return launch_tc<192, tc::RESID_WIDE, 64>(c, A, W, M, N, K, epi);
+    if (ek == tc::RESID_HALF) return launch_tc<192, tc::RESID_HALF, 64>(c, A, W, M, N, K, epi);
+    return launch_tc<192, tc::BF16OUT, 64>(c, A, W, M, N, K, epi);
   }
   if (bn == 256) {
-    if (ek == tc::RESID_WIDE) return launch_tc<256, tc::RESID_WIDE>(c, A, W, M, N, K, epi);
-    if (ek == tc::RESID_HALF) return launch_tc<256, tc::RESID_HALF>(c, A, W, M, N, K, epi);
-    return launch_tc<256, tc::BF16OUT>(c, A, W, M, N, K, epi);
+    if (ek == tc::RESID_WIDE) return launch_tc<256, tc::RESID_WIDE, 64>(c, A, W, M, N, K, epi);
+    if (ek == tc::RESID_HALF) return launch_tc<256, tc::RESID_HALF, 64>(c, A, W, M, N, K, epi);
+    return launch_tc<256, tc::BF16OUT, 64>(c, A, W, M, N, K, epi);
   }
-  if (ek == tc::RESID_WIDE) return launch_tc<128, tc::RESID_WIDE>(c, A, W, M, N, K, epi);
-  if (ek == tc::RESID_HALF) return launch_tc<128, tc::RESID_HALF>(c, A, W, M, N, K, epi);
-  return launch_tc<128, tc::BF16OUT>(c, A, W, M, N, K, epi);
+  if (K % 128 == 0) {
+    if (ek == tc::RESID_WIDE) return launch_tc<128, tc::RESID_WIDE, 128>(c, A, W, M, N, K, epi);
+    if (ek == tc::RESID_HALF) return launch_tc<128, tc::RESID_HALF, 128>(c, A, W, M, N, K, epi);
+    return launch_tc<128, tc::BF16OUT, 128>(c, A, W, M, N, K, epi);
+  }
+  if (ek == tc::RESID_WIDE) return launch_tc<128, tc::RESID_WIDE, 64>(c, A, W, M, N, K, epi);
+  if (ek == tc::RESID_HALF) return launch_tc<128, tc::RESID_HALF, 64>(c, A, W, M, N, K, epi);
+  return launch_tc<128, tc::BF16OUT, 64>(c, A, W, M, N, K, epi);
 }
 
 }  // namespace lm

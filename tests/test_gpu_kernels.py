@@ -132,6 +132,7 @@ def test_cfg_combine(dtype, mode, n):
 GEMM_SHAPES = [
     (1, 384, 128), (40, 768, 256), (200, 2304, 768), (3200, 2304, 768), (3200, 768, 768),
     (3200, 3072, 768), (3200, 768, 3072), (777, 1280, 1280), (384, 3840, 1280),
+    (100, 256, 192), (33, 384, 320),  # K not a multiple of 128: 64-deep stages at every width
 ]
 
 
