@@ -59,7 +59,7 @@ def peaks():
 NAMES = {"mar_b": "MAR-B", "mar_l": "MAR-L", "mar_h": "MAR-H", "hires": "MAR-L high-resolution", "tiny": "tiny"}
 
 
-def workload(cfg):
+def workload(cfg, select="least_similar"):
     n = synth.n_compute(cfg)
     return {
         "workload": "%s-shaped %d-step LazyMAR decode (%d blocks, width %d, %d heads, %d+%d tokens)" % (
@@ -71,6 +71,7 @@ def workload(cfg):
             cfg["k0"], cfg["tau"], "no condition cache" if cfg["tau_cfg"] == 0 else
             "cond cache reused on cached steps with (k-k0) %% %d != 0" % cfg["tau_cfg"]),
         "decoding_steps": cfg["steps"],
+        "selection": select,
         "l2": "no flush: the per-step working set (%.2f GB weights + %.2f GB K/V cache) exceeds the 129 MB L2" % (
             12 * cfg["depth"] * cfg["width"] ** 2 * 2 / 1e9,
             2 * (cfg["depth"] - cfg["sel_layers"]) * 2 * cfg["batch"] * cfg["T"] * cfg["width"] * 2 / 1e9),
@@ -79,6 +80,31 @@ def workload(cfg):
 
 def schedule(cfg, plan_fn):
     return [plan_fn(k, cfg["k0"], cfg["tau"], cfg["tau_cfg"], True) for k in range(cfg["steps"])]
+
+
+SELECT_RULES = {"least_similar": 0, "most_similar": 1, "random": 2, "observation": 0}
+
+
+def selection_inputs(cfg, masks, rule_name, seed_offset):
+    """Per-step selection inputs of the Table 3 strategies for [2B, T] rows (a
+    cond-reuse step uses the first B): random keys (strategy III, seeded) or
+    observation-based priorities (1 for the image tokens decoded at the
+    previous step and at this step, Sec. 3.2.1); None where unused."""
+    steps, B, n_img = masks.shape
+    T, nb = cfg["T"], cfg["n_buffer"]
+    if rule_name == "random":
+        rng = np.random.default_rng(4 + seed_offset)
+        return None, rng.integers(0, 1 << 32, size=(steps, 2 * B, T), dtype=np.uint64).astype(np.uint32)
+    if rule_name != "observation":
+        return None, None
+    prio = np.zeros((steps, 2 * B, T), np.uint8)
+    for k in range(steps):
+        prev = masks[k - 1] if k > 0 else np.ones_like(masks[0])
+        nxt = masks[k + 1] if k + 1 < steps else np.zeros_like(masks[0])
+        hot = ((prev != 0) & (masks[k] == 0)) | ((masks[k] != 0) & (nxt == 0))
+        prio[k, :B, nb:] = hot
+        prio[k, B:, nb:] = hot
+    return prio, None
 
 
 def decode_inputs(cfg, seed_offset):
@@ -207,7 +233,7 @@ def run_reference(args, cfg, plan):
     cb.pop("sample_s", None)
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "images/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 / value, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": workload(cfg),
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": workload(cfg, args.select),
             "cpu_baseline": cb, "e2e": {"value": value, "unit": "images/s", "h2d_bytes_per_step": 0,
                                         "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -239,27 +265,32 @@ def run_ours(args, cfg):
 
     B, N, steps = cfg["batch"], synth.n_compute(cfg), cfg["steps"]
     W = synth.make_weights(cfg)
-    h = lm.lazymar_create(dict(cfg, max_batch=B), W)
+    h = lm.lazymar_create(dict(cfg, max_batch=B, select_rule=SELECT_RULES[args.select]), W)
     lat_np, mask_np, labels_np = decode_inputs(cfg, rank * 101)
     lat = torch.from_numpy(lat_np).cuda()
     mask = torch.from_numpy(mask_np).cuda()
     labels = torch.from_numpy(labels_np).cuda()
+    prio_np, keys_np = selection_inputs(cfg, mask_np, args.select, rank * 101)
+    prio = None if prio_np is None else torch.from_numpy(prio_np).cuda()
+    keys = None if keys_np is None else torch.from_numpy(keys_np.view(np.int32)).cuda()
     guided = torch.empty((B, cfg["n_img"], cfg["width"]), dtype=torch.bfloat16, device="cuda")
     stream = torch.cuda.current_stream()
+    dev_in = {"lat": lat, "mask": mask, "labels": labels, "guided": guided, "prio": prio, "keys": keys}
 
     def decode(full_only=False, host=None, step_events=None):
         for k in range(steps):
             full, reuse = plan[k]
-            if host is not None:
-                l_k, m_k, lab, g = host["lat"][k], host["mask"][k], host["labels"], host["guided"]
-            else:
-                l_k, m_k, lab, g = lat[k], mask[k], labels, guided
+            src = host if host is not None else dev_in
+            l_k, m_k, lab, g = src["lat"][k], src["mask"][k], src["labels"], src["guided"]
+            p_k = None if src["prio"] is None else src["prio"][k]
+            r_k = None if src["keys"] is None else src["keys"][k]
             if step_events is not None:
                 step_events[k][0].record(stream)
             if full or full_only:
                 lm.lazymar_full_step(h, l_k, m_k, lab, B, GAMMA, None, g, stream)
             else:
-                lm.lazymar_cached_step(h, l_k, m_k, lab, B, N, reuse, GAMMA, None, None, None, g, stream)
+                lm.lazymar_cached_step(h, l_k, m_k, lab, B, N, reuse, GAMMA, None, None, None, g, stream,
+                                       select_priority=p_k, select_keys=r_k)
             if step_events is not None:
                 step_events[k][1].record(stream)
         if host is not None:
@@ -323,11 +354,16 @@ def run_ours(args, cfg):
 
     # 4) end to end through the C ABI with host buffers (pinned), copies inside
     host = {"lat": lat.cpu().pin_memory(), "mask": mask.cpu().pin_memory(), "labels": labels.cpu().pin_memory(),
-            "guided": torch.empty(tuple(guided.shape), dtype=torch.bfloat16).pin_memory()}
+            "guided": torch.empty(tuple(guided.shape), dtype=torch.bfloat16).pin_memory(),
+            "prio": None if prio is None else prio.cpu().pin_memory(),
+            "keys": None if keys is None else keys.cpu().pin_memory()}
     decode(host=host)
     ms_e2e, _ = timed(lambda: decode(host=host), args.steps)
     e2e_images_per_s = world * B * args.steps / (ms_e2e / 1000.0)
-    h2d = steps * (lat[0].numel() * 4 + mask[0].numel() + labels.numel() * 4)
+    # selection inputs are copied on cached steps only, for the rows they run
+    cached_rows = sum(0 if f else (B if r else 2 * B) for f, r in plan)
+    sel_bytes = cached_rows * cfg["T"] * ((1 if prio is not None else 0) + (4 if keys is not None else 0))
+    h2d = steps * (lat[0].numel() * 4 + mask[0].numel() + labels.numel() * 4) + sel_bytes
     d2h = steps * guided.numel() * 2
     lm.lazymar_sync(h, stream)
 
@@ -358,7 +394,7 @@ def run_ours(args, cfg):
         "metric": METRIC, "value": images_per_s, "unit": "images/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded latents/masks, random-init MAR-B weights)",
-        "config": workload(cfg),
+        "config": workload(cfg, args.select),
         "decoding_steps_per_s": world * steps * args.steps / (ms / 1000.0),
         "step_ms": {k: round(statistics.mean(v), 3) for k, v in kind_ms.items() if v},
         "full_recompute": {"value": full_images_per_s, "unit": "images/s", "ms_per_step": ms_full / args.steps,
@@ -434,6 +470,8 @@ def main():
     ap.add_argument("--config", default="mar_b")
     ap.add_argument("--ratio", type=float, default=None, help="recompute ratio (default: the config's)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--select", default="least_similar", choices=sorted(SELECT_RULES),
+                    help="token-selection strategy of the cached steps (Table 3; default: LazyMAR's)")
     ap.add_argument("--profile-case", choices=["gemm_layers", "attention_layers"], default=None,
                     help="run each kernel of a layer once at the configuration's shapes (for ncu) and exit")
     args = ap.parse_args()

@@ -71,6 +71,24 @@ typedef enum lazymar_criterion {
   LAZYMAR_CRITERION_FEATURE = 1
 } lazymar_criterion;
 
+/* Which tokens fill the recompute budget N of a cached step (Sec. 4.4,
+ * Table 3 "token selection strategies"). LEAST_SIMILAR: the N tokens least
+ * similar to their cached values (strategy V, LazyMAR's default; recompute
+ * least similar = cache most similar). MOST_SIMILAR: the N most similar
+ * (strategy IV: cache the minimum-similarity tokens). RANDOM: the N tokens
+ * with the smallest caller-drawn 32-bit keys (strategy III; the random draw is
+ * an input). Ties go to the lower token index; a NaN similarity counts as
+ * -inf. An optional per-token priority class (uint8, higher first) is applied
+ * before the rule: it expresses the strategies that choose by token type, for
+ * example the observation-based strategy of Sec. 3.2.1 (priority 1 for tokens
+ * decoded at steps t-1 and t) or strategies I/II (priority 1 for decoded,
+ * respectively still-masked, tokens). */
+typedef enum lazymar_select_rule {
+  LAZYMAR_SELECT_LEAST_SIMILAR = 0,
+  LAZYMAR_SELECT_MOST_SIMILAR = 1,
+  LAZYMAR_SELECT_RANDOM = 2
+} lazymar_select_rule;
+
 /* Model and capacity. width % 128 == 0, head width (width/heads) 64 or 80 for
  * bf16 (any divisor of width up to 128 for f32), token_dim <= 64,
  * 1 <= sel_layers <= depth, 1 <= max_batch (pairs). */
@@ -88,6 +106,7 @@ typedef struct lazymar_config {
   int dtype;       /* lazymar_dtype of weights, activations and caches */
   int criterion;   /* lazymar_criterion */
   float ln_eps;    /* LayerNorm epsilon */
+  int select_rule; /* lazymar_select_rule of the cached steps (0 = strategy V) */
 } lazymar_config;
 
 /* Weights of one pre-LN block, fp32, [out, in] layout (y = x W^T + b).
@@ -112,12 +131,17 @@ typedef struct lazymar_weights {
   const lazymar_block_weights *blocks;   /* host array of `depth` entries */
 } lazymar_weights;
 
-/* Inputs of one decoding step for B pairs (both pathways share them). */
+/* Inputs of one decoding step for B pairs (both pathways share them). The two
+ * selection inputs are read by cached steps only, for the rows that step runs
+ * (2B, or B when it reuses the condition cache), and may be NULL (RANDOM
+ * requires select_keys). */
 typedef struct lazymar_step_in {
   const float *latents;   /* [B, n_img, token_dim] fp32; ignored where masked */
   const uint8_t *mask;    /* [B, n_img], 1 = still masked, 0 = decoded */
   const int32_t *labels;  /* [B] class labels in [0, n_classes) */
   int batch;              /* B, 1 <= B <= max_batch */
+  const uint8_t *select_priority; /* [rows, T] priority classes, higher recomputed first */
+  const uint32_t *select_keys;    /* [rows, T] random keys of LAZYMAR_SELECT_RANDOM */
 } lazymar_step_in;
 
 typedef struct lazymar_handle lazymar_handle;
@@ -170,6 +194,17 @@ lazymar_status lazymar_cached_step(lazymar_handle *h, const lazymar_step_in *in,
  * Allocates rows*T doubles of stream-ordered scratch (cudaMallocAsync). */
 lazymar_status lazymar_select_tokens(int dtype, const void *v_cur, void *v_cache, int rows, int T,
                                      int D, int n_compute, int32_t *idx_out, void *stream);
+
+/* lazymar_select_tokens under a selection rule (lazymar_select_rule, Table 3)
+ * with optional per-token priority classes: tokens are taken by priority
+ * descending, then the rule, then index ascending. priority [rows, T] uint8
+ * may be NULL; keys [rows, T] uint32 are required for LAZYMAR_SELECT_RANDOM
+ * and ignored otherwise. The similarities are computed and v_cache := v_cur
+ * under every rule. Device pointers only; same scratch as
+ * lazymar_select_tokens. */
+lazymar_status lazymar_select_tokens_ex(int dtype, const void *v_cur, void *v_cache, int rows, int T,
+                                        int D, int n_compute, int rule, const uint8_t *priority,
+                                        const uint32_t *keys, int32_t *idx_out, void *stream);
 
 /* lazymar_select_tokens without any device allocation. The paper has no
  * counterpart: this entry point exists for callers that may not allocate

@@ -177,6 +177,41 @@ def select_compute(S, n):
     return np.sort(order[:n]).astype(np.int64)
 
 
+# Token-selection rules (Table 3): which tokens fill the recompute budget N.
+SELECT_LEAST_SIMILAR = 0  # strategy V (LazyMAR): cache the most similar, recompute the least
+SELECT_MOST_SIMILAR = 1   # strategy IV: cache the least similar, recompute the most
+SELECT_RANDOM = 2         # strategy III: caller-drawn random priority keys
+
+
+def select_by_rule(S, n, rule=SELECT_LEAST_SIMILAR, priority=None, keys=None):
+    """I_compute for one row under the selection strategies of Sec. 4.4 (Table 3)
+    and the observation-based strategy of Sec. 3.2.1.
+
+    Tokens are taken in the order: priority descending (when given), then the
+    rule, then token index ascending; the first n are recomputed, returned
+    ascending. Rules: SELECT_LEAST_SIMILAR, S ascending (strategy V, the
+    default, equal to select_compute); SELECT_MOST_SIMILAR, S descending
+    (strategy IV); SELECT_RANDOM, ascending `keys` (strategy III: the random
+    draw is an input). A NaN S counts as -inf under both similarity rules.
+    Reading: the priority classes express the strategies that choose by token
+    type. Observation-based: 1 for tokens decoded at step t-1 or decoded at
+    step t, which are always recomputed. Strategy I (cache the unpredicted
+    tokens): 1 for decoded tokens. Strategy II (cache the predicted tokens): 1
+    for masked tokens. The paper gives no order inside a class; the rule
+    decides.
+    """
+    S = np.asarray(S, F64)
+    T = S.shape[0]
+    if rule == SELECT_RANDOM:
+        key = np.asarray(keys, np.int64)
+    else:
+        Sm = np.where(np.isnan(S), -np.inf, S)
+        key = Sm if rule == SELECT_LEAST_SIMILAR else -Sm
+    prio = np.zeros(T, np.int64) if priority is None else np.asarray(priority, np.int64)
+    order = np.lexsort((np.arange(T), key, -prio))
+    return np.sort(order[:n]).astype(np.int64)
+
+
 # ----------------------------------------------------------------------------
 # Classifier-free guidance and the condition cache (Eq. 7, Eq. 10)
 # ----------------------------------------------------------------------------
@@ -285,7 +320,8 @@ def full_step(cfg, W, cache, latents, mask, labels, gamma):
     return z, guidance(z[:B], z[B:], gamma)
 
 
-def cached_step(cfg, W, cache, latents, mask, labels, n, cond_reuse, gamma, idx=None):
+def cached_step(cfg, W, cache, latents, mask, labels, n, cond_reuse, gamma, idx=None, rule=SELECT_LEAST_SIMILAR,
+                priority=None, keys=None):
     """A cached step: token cache (Eq. 8, Eq. 9) and optionally the condition cache.
 
     Blocks 0..s-1 run over all tokens (the paper's "first three layers"). At
@@ -300,6 +336,8 @@ def cached_step(cfg, W, cache, latents, mask, labels, n, cond_reuse, gamma, idx=
     rebuilt as c - delta (Sec. 3.2.2). Otherwise both pathways run and the
     condition cache is refreshed.
     idx: optional [rows, N] caller-chosen I_compute (used instead of Eq. 8).
+    rule, priority [rows, T], keys [rows, T]: the selection strategy of
+    select_by_rule (default: strategy V, the N least similar tokens).
 
     Returns z [2B, n_img, D], guided [B, n_img, D], I_compute [rows, N] and the
     similarities S [rows, T].
@@ -320,7 +358,10 @@ def cached_step(cfg, W, cache, latents, mask, labels, n, cond_reuse, gamma, idx=
             x = x_new
         S = cosine_similarity(cur, cache.ref[r])
         cache.ref[r] = cur
-        I = select_compute(S, n) if idx is None else np.asarray(idx[r], np.int64)
+        if idx is not None:
+            I = np.asarray(idx[r], np.int64)
+        else:
+            I = select_by_rule(S, n, rule, None if priority is None else priority[r], None if keys is None else keys[r])
         xs = x[I]
         for l in range(s, L):
             xs = block_cached(W["blocks"][l], xs, I, cache.K[l][r], cache.V[l][r], H, eps)

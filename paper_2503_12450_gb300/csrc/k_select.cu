@@ -222,25 +222,54 @@ __device__ __forceinline__ unsigned long long sim_key(double s) {
   return (u >> 63) ? ~u : (u | 0x8000000000000000ull);
 }
 
+// Selection order (Table 3 strategies): priority descending when given, then
+// the rule's key ascending, then token index. Keys: LEAST_SIMILAR (strategy V)
+// the order-preserving key of S; MOST_SIMILAR (strategy IV) its complement,
+// i.e. S descending (NaN, as -inf, last); RANDOM (strategy III) the caller's
+// 32-bit random keys.
 __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const double* __restrict__ S, int T, int N,
-                                                            int* __restrict__ idx, int* __restrict__ row_map) {
-  extern __shared__ unsigned long long sK[];  // T keys
+                                                            int* __restrict__ idx, int* __restrict__ row_map,
+                                                            int rule, const uint8_t* __restrict__ prio,
+                                                            const uint32_t* __restrict__ rkeys) {
+  extern __shared__ unsigned long long sK[];  // T keys, then T priorities, then T flags
   __shared__ int s_wcount[kTopkThreads / 32];
   __shared__ int s_woff[kTopkThreads / 32];
   __shared__ int s_total;
-  unsigned char* sel = reinterpret_cast<unsigned char*>(sK + T);
+  unsigned char* sP = reinterpret_cast<unsigned char*>(sK + T);
+  unsigned char* sel = sP + T;
   const int r = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   pdl_wait();
   pdl_trigger();
-  for (int t = tid; t < T; t += kTopkThreads) sK[t] = sim_key(S[(size_t)r * T + t]);
+  for (int t = tid; t < T; t += kTopkThreads) {
+    const size_t i = (size_t)r * T + t;
+    unsigned long long k;
+    if (rule == LAZYMAR_SELECT_RANDOM) {
+      k = rkeys[i];
+    } else {
+      k = sim_key(S[i]);
+      if (rule == LAZYMAR_SELECT_MOST_SIMILAR) k = ~k;
+    }
+    sK[t] = k;
+    sP[t] = prio ? prio[i] : 0;
+  }
   __syncthreads();
-  // rank of token t under (S ascending, index ascending); I_compute = rank < N
+  // rank of token t under (priority descending, key ascending, index
+  // ascending); I_compute = rank < N
   for (int t = tid; t < T; t += kTopkThreads) {
     const unsigned long long kt = sK[t];
+    const unsigned pt = sP[t];
     int rank = 0;
-    for (int u = 0; u < T; ++u) {
-      const unsigned long long ku = sK[u];
-      rank += (ku < kt) || (ku == kt && u < t);
+    if (prio) {
+      for (int u = 0; u < T; ++u) {
+        const unsigned long long ku = sK[u];
+        const unsigned pu = sP[u];
+        rank += (pu > pt) || (pu == pt && ((ku < kt) || (ku == kt && u < t)));
+      }
+    } else {
+      for (int u = 0; u < T; ++u) {
+        const unsigned long long ku = sK[u];
+        rank += (ku < kt) || (ku == kt && u < t);
+      }
     }
     sel[t] = rank < N;
   }
@@ -274,14 +303,16 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const double* __rest
   }
 }
 
-cudaError_t launch_topk(const Ctx& c, const double* S, int rows, int T, int N, int* idx, int* row_map) {
+cudaError_t launch_topk(const Ctx& c, const double* S, int rows, int T, int N, int* idx, int* row_map, int rule,
+                        const uint8_t* prio, const uint32_t* keys) {
   if (rows == 0 || N == 0) return cudaSuccess;
-  const size_t smem = (size_t)T * sizeof(unsigned long long) + (size_t)T;
+  const size_t smem = (size_t)T * sizeof(unsigned long long) + 2 * (size_t)T;
   if (smem > 48 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
   }
-  return launch_pdl(topk_kernel, dim3(rows), dim3(kTopkThreads), smem, c.stream, S, T, N, idx, row_map);
+  return launch_pdl(topk_kernel, dim3(rows), dim3(kTopkThreads), smem, c.stream, S, T, N, idx, row_map, rule, prio,
+                    keys);
 }
 
 // Caller-chosen I_compute: copied after checking range and strict increase per

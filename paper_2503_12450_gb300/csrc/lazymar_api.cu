@@ -114,6 +114,8 @@ struct lazymar_handle {
   float* st_lat = nullptr;
   uint8_t* st_mask = nullptr;
   int *st_labels = nullptr, *st_idx_in = nullptr, *st_idx_out = nullptr;
+  uint8_t* st_prio = nullptr;     // [rows, T] selection priority classes
+  uint32_t* st_keys = nullptr;    // [rows, T] selection random keys
   void *st_z = nullptr, *st_g = nullptr;
   unsigned* err = nullptr;
   bool primed = false;
@@ -129,9 +131,9 @@ struct lazymar_handle {
   size_t ev_used = 0;
   // CUDA graphs of step bodies, keyed by (kind, batch, N, cond reuse, caller indices)
   struct GraphKey {
-    int kind, B, N, reuse, idx;
+    int kind, B, N, reuse, idx, sel;  // sel: bit 0 priority given, bit 1 keys given
     bool operator<(const GraphKey& o) const {
-      return std::tie(kind, B, N, reuse, idx) < std::tie(o.kind, o.B, o.N, o.reuse, o.idx);
+      return std::tie(kind, B, N, reuse, idx, sel) < std::tie(o.kind, o.B, o.N, o.reuse, o.idx, o.sel);
     }
   };
   struct GraphEntry {
@@ -228,6 +230,8 @@ lazymar_status check_config(const lazymar_config* c) {
   if (c->dtype != LAZYMAR_F32 && c->dtype != LAZYMAR_BF16) return fail(LAZYMAR_ERR_INVALID_ARG, "config: dtype");
   if (c->criterion != LAZYMAR_CRITERION_VALUE && c->criterion != LAZYMAR_CRITERION_FEATURE)
     return fail(LAZYMAR_ERR_INVALID_ARG, "config: criterion");
+  if (c->select_rule < LAZYMAR_SELECT_LEAST_SIMILAR || c->select_rule > LAZYMAR_SELECT_RANDOM)
+    return fail(LAZYMAR_ERR_INVALID_ARG, "config: select_rule");
   if (c->sel_layers < 1 || c->sel_layers > c->depth)
     return fail(LAZYMAR_ERR_INVALID_ARG, "config: 1 <= sel_layers <= depth required");
   if (c->token_dim < 1 || c->token_dim > 64) return fail(LAZYMAR_ERR_UNSUPPORTED, "config: token_dim must be 1..64");
@@ -295,6 +299,7 @@ extern "C" lazymar_status lazymar_create(const lazymar_config* cfg, const lazyma
   // staging
   const size_t o_lat = b.take(Bm * cfg->n_img * cfg->token_dim * 4), o_mask = b.take(Bm * cfg->n_img),
                o_lab = b.take(Bm * 4), o_iin = b.take(rowsT * 4), o_iout = b.take(rowsT * 4),
+               o_prio = b.take(rowsT), o_keys = b.take(rowsT * 4),
                o_stz = b.take(R * cfg->n_img * D * es), o_stg = b.take(Bm * cfg->n_img * D * es),
                o_err = b.take(sizeof(unsigned));
   h->arena_bytes = b.off;
@@ -333,6 +338,7 @@ extern "C" lazymar_status lazymar_create(const lazymar_config* cfg, const lazyma
   h->st_lat = reinterpret_cast<float*>(a + o_lat); h->st_mask = a + o_mask;
   h->st_labels = reinterpret_cast<int*>(a + o_lab);
   h->st_idx_in = reinterpret_cast<int*>(a + o_iin); h->st_idx_out = reinterpret_cast<int*>(a + o_iout);
+  h->st_prio = a + o_prio; h->st_keys = reinterpret_cast<uint32_t*>(a + o_keys);
   h->st_z = a + o_stz; h->st_g = a + o_stg;
   h->err = reinterpret_cast<unsigned*>(a + o_err);
 
@@ -520,7 +526,7 @@ lazymar_status full_body(lazymar_handle* h, const Ctx& c, int B) {
 }
 
 // Device work of a cached step up to the output cache.
-lazymar_status cached_body(lazymar_handle* h, const Ctx& c, int rows, int N, bool has_idx) {
+lazymar_status cached_body(lazymar_handle* h, const Ctx& c, int rows, int N, bool has_idx, int sel) {
   const int s = h->s, T = h->T, D = h->D;
   LM_TRY(embed(h, c, rows, h->last_batch));
   for (int l = 0; l < s; ++l) LM_TRY(layer_full(h, c, l, rows, h->Ks, h->Vs));
@@ -540,7 +546,10 @@ lazymar_status cached_body(lazymar_handle* h, const Ctx& c, int rows, int N, boo
                   [&] { return launch_idx_check(c, h->st_idx_in, rows, T, N, h->idx, h->row_map); }));
   } else if (N > 0) {
     LM_TRY(launch(h, LAZYMAR_K_SELECT, 0, 8.0 * rows * T + 8.0 * rows * N, c.stream, "topk",
-                  [&] { return launch_topk(c, h->S, rows, T, N, h->idx, h->row_map); }));
+                  [&] {
+                    return launch_topk(c, h->S, rows, T, N, h->idx, h->row_map, h->cfg.select_rule,
+                                       (sel & 1) ? h->st_prio : nullptr, (sel & 2) ? h->st_keys : nullptr);
+                  }));
   }
   if (N > 0) {
     for (int l = s; l < h->L; ++l) LM_TRY(layer_cached(h, c, l, rows, N, l == s));
@@ -609,7 +618,7 @@ extern "C" lazymar_status lazymar_full_step(lazymar_handle* h, const lazymar_ste
   const Ctx c{st, h->err, h->num_sms};
   const int B = in->batch;
   LM_TRY(stage_inputs(h, in, st));
-  LM_TRY(run_body(h, st, lazymar_handle::GraphKey{0, B, 0, 0, 0}, [&](const Ctx& cc) { return full_body(h, cc, B); }));
+  LM_TRY(run_body(h, st, lazymar_handle::GraphKey{0, B, 0, 0, 0, 0}, [&](const Ctx& cc) { return full_body(h, cc, B); }));
   void* g_dst = out_target(guided_out, h->st_g);
   LM_TRY(cfg(h, c, LAZYMAR_CFG_REFRESH, B, gamma, nullptr, g_dst));
   const size_t zbytes = (size_t)2 * B * h->cfg.n_img * h->D * h->es;
@@ -635,8 +644,18 @@ extern "C" lazymar_status lazymar_cached_step(lazymar_handle* h, const lazymar_s
   LM_TRY(stage_inputs(h, in, st));
   const bool has_idx = idx_in != nullptr && N > 0;
   if (has_idx) LM_CUDA(cudaMemcpyAsync(h->st_idx_in, idx_in, (size_t)rows * N * 4, cudaMemcpyDefault, st));
-  LM_TRY(run_body(h, st, lazymar_handle::GraphKey{1, B, N, use_cond_cache ? 1 : 0, has_idx ? 1 : 0},
-                  [&](const Ctx& cc) { return cached_body(h, cc, rows, N, has_idx); }));
+  // selection inputs (Table 3 rules): priority classes and random keys
+  const bool sel_rule = !has_idx && N > 0;
+  const bool has_prio = sel_rule && in->select_priority != nullptr;
+  const bool has_keys = sel_rule && h->cfg.select_rule == LAZYMAR_SELECT_RANDOM;
+  if (has_keys && !in->select_keys)
+    return fail(LAZYMAR_ERR_INVALID_ARG, "LAZYMAR_SELECT_RANDOM needs select_keys on cached steps");
+  const size_t rowsT = (size_t)rows * h->T;
+  if (has_prio) LM_CUDA(cudaMemcpyAsync(h->st_prio, in->select_priority, rowsT, cudaMemcpyDefault, st));
+  if (has_keys) LM_CUDA(cudaMemcpyAsync(h->st_keys, in->select_keys, rowsT * 4, cudaMemcpyDefault, st));
+  const int sel = (has_prio ? 1 : 0) | (has_keys ? 2 : 0);
+  LM_TRY(run_body(h, st, lazymar_handle::GraphKey{1, B, N, use_cond_cache ? 1 : 0, has_idx ? 1 : 0, sel},
+                  [&](const Ctx& cc) { return cached_body(h, cc, rows, N, has_idx, sel); }));
 
   const size_t n_el = (size_t)B * h->cfg.n_img * D;
   void* z_dst = out_target(z_out, h->st_z);
@@ -665,25 +684,38 @@ extern "C" lazymar_status lazymar_set_graphs(lazymar_handle* h, int enable) {
 // ---------------------------------------------------------------------------
 // Component entry points
 // ---------------------------------------------------------------------------
-extern "C" lazymar_status lazymar_select_tokens(int dtype, const void* v_cur, void* v_cache, int rows, int T, int D,
-                                                int n_compute, int32_t* idx_out, void* stream) {
+extern "C" lazymar_status lazymar_select_tokens_ex(int dtype, const void* v_cur, void* v_cache, int rows, int T,
+                                                   int D, int n_compute, int rule, const uint8_t* priority,
+                                                   const uint32_t* keys, int32_t* idx_out, void* stream) {
   if (dtype != LAZYMAR_F32 && dtype != LAZYMAR_BF16) return fail(LAZYMAR_ERR_INVALID_ARG, "dtype");
+  if (rule < LAZYMAR_SELECT_LEAST_SIMILAR || rule > LAZYMAR_SELECT_RANDOM) return fail(LAZYMAR_ERR_INVALID_ARG, "rule");
   if (rows < 0 || T < 1 || T > 16384 || D < 8 || D % 8 != 0 || n_compute < 0 || n_compute > T)
     return fail(LAZYMAR_ERR_INVALID_ARG, "rows >= 0, 1 <= T <= 16384, D % 8 == 0, 0 <= n_compute <= T required");
   if (rows == 0) return LAZYMAR_OK;
   if (!is_device_ptr(v_cur) || !is_device_ptr(v_cache) || (n_compute > 0 && !is_device_ptr(idx_out)))
     return fail(LAZYMAR_ERR_INVALID_ARG, "v_cur, v_cache and idx_out must be device pointers");
+  if (priority && !is_device_ptr(priority)) return fail(LAZYMAR_ERR_INVALID_ARG, "priority must be a device pointer");
+  if (rule == LAZYMAR_SELECT_RANDOM && !is_device_ptr(keys))
+    return fail(LAZYMAR_ERR_INVALID_ARG, "LAZYMAR_SELECT_RANDOM needs device keys");
   if (!aligned16(v_cur) || !aligned16(v_cache)) return fail(LAZYMAR_ERR_INVALID_ARG, "16-byte alignment required");
   Ctx c;
   LM_TRY(component_ctx(stream, &c));
   double* S = nullptr;
   LM_CUDA(cudaMallocAsync(reinterpret_cast<void**>(&S), (size_t)rows * T * sizeof(double), c.stream));
   cudaError_t e = launch_similarity(c, dtype, v_cur, v_cache, S, rows, T, D, true);
-  if (e == cudaSuccess) e = launch_topk(c, S, rows, T, n_compute, idx_out, nullptr);
+  if (e == cudaSuccess)
+    e = launch_topk(c, S, rows, T, n_compute, idx_out, nullptr, rule, priority,
+                    rule == LAZYMAR_SELECT_RANDOM ? keys : nullptr);
   cudaError_t e2 = cudaFreeAsync(S, c.stream);
   if (e != cudaSuccess) return cuda_fail(e, "select kernels");
   if (e2 != cudaSuccess) return cuda_fail(e2, "cudaFreeAsync");
   return LAZYMAR_OK;
+}
+
+extern "C" lazymar_status lazymar_select_tokens(int dtype, const void* v_cur, void* v_cache, int rows, int T, int D,
+                                                int n_compute, int32_t* idx_out, void* stream) {
+  return lazymar_select_tokens_ex(dtype, v_cur, v_cache, rows, T, D, n_compute, LAZYMAR_SELECT_LEAST_SIMILAR, nullptr,
+                                  nullptr, idx_out, stream);
 }
 
 extern "C" lazymar_status lazymar_cfg_combine(int dtype, int mode, const void* z_cond, const void* z_uncond,

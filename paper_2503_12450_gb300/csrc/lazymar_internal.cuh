@@ -388,7 +388,8 @@ cudaError_t launch_cast(const Ctx& c, int dtype, const float* x, void* y, size_t
 
 cudaError_t launch_similarity(const Ctx& c, int dtype, const void* cur, void* cache, double* S, int rows, int T,
                               int D, bool copy);
-cudaError_t launch_topk(const Ctx& c, const double* S, int rows, int T, int N, int* idx, int* row_map);
+cudaError_t launch_topk(const Ctx& c, const double* S, int rows, int T, int N, int* idx, int* row_map,
+                        int rule = 0, const uint8_t* prio = nullptr, const uint32_t* keys = nullptr);
 cudaError_t launch_idx_check(const Ctx& c, const int* idx_in, int rows, int T, int N, int* idx, int* row_map);
 cudaError_t launch_cfg(const Ctx& c, int dtype, int mode, const void* zc, const void* zu, void* delta,
                        float gamma, size_t n, void* zu_out, void* g_out);

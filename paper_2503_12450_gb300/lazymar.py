@@ -14,6 +14,7 @@ LIB_PATH = os.path.join(HERE, "liblazymar.so")
 
 LAZYMAR_F32, LAZYMAR_BF16 = 0, 1
 LAZYMAR_CRITERION_VALUE, LAZYMAR_CRITERION_FEATURE = 0, 1
+LAZYMAR_SELECT_LEAST_SIMILAR, LAZYMAR_SELECT_MOST_SIMILAR, LAZYMAR_SELECT_RANDOM = 0, 1, 2
 LAZYMAR_CFG_GUIDE, LAZYMAR_CFG_REFRESH, LAZYMAR_CFG_REUSE = 0, 1, 2
 LAZYMAR_EPI_BIAS, LAZYMAR_EPI_GELU, LAZYMAR_EPI_RESIDUAL, LAZYMAR_EPI_QKV = 0, 1, 2, 3
 KERNEL_CLASSES = ["gemm", "attention", "layernorm", "select", "embed", "cfg", "other"]
@@ -30,7 +31,7 @@ class LazymarError(RuntimeError):
 class lazymar_config(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int) for n in ("depth", "width", "heads", "mlp_ratio", "n_buffer", "n_img", "token_dim",
                                              "n_classes", "max_batch", "sel_layers", "dtype", "criterion")] + [
-        ("ln_eps", ctypes.c_float)]
+        ("ln_eps", ctypes.c_float), ("select_rule", ctypes.c_int)]
 
 
 _FP = ctypes.c_void_p
@@ -47,7 +48,8 @@ class lazymar_weights(ctypes.Structure):
 
 
 class lazymar_step_in(ctypes.Structure):
-    _fields_ = [("latents", _FP), ("mask", _FP), ("labels", _FP), ("batch", ctypes.c_int)]
+    _fields_ = [("latents", _FP), ("mask", _FP), ("labels", _FP), ("batch", ctypes.c_int),
+                ("select_priority", _FP), ("select_keys", _FP)]
 
 
 class lazymar_kernel_stats(ctypes.Structure):
@@ -79,6 +81,7 @@ def lib():
         "lazymar_cached_step": (st, [vp, ctypes.POINTER(lazymar_step_in), i, i, f, vp, vp, vp, vp, vp]),
         "lazymar_select_tokens": (st, [i, vp, vp, i, i, i, i, vp, vp]),
         "lazymar_select_tokens_noalloc": (st, [i, vp, vp, i, i, i, i, vp, vp]),
+        "lazymar_select_tokens_ex": (st, [i, vp, vp, i, i, i, i, i, vp, vp, vp, vp]),
         "lazymar_cfg_combine": (st, [i, i, vp, vp, vp, f, sz, vp, vp, vp]),
         "lazymar_linear": (st, [i, i, vp, vp, vp, i, i, i, vp, i, vp, vp, vp, i, vp]),
         "lazymar_attention": (st, [i, vp, vp, vp, vp, i, i, i, i, i, vp]),
@@ -140,7 +143,7 @@ def lazymar_create(cfg, weights):
     arrays or torch tensors as produced by synth.make_weights. Returns a Handle."""
     c = lazymar_config()
     for n, _ in lazymar_config._fields_:
-        if n in ("dtype", "criterion", "ln_eps"):
+        if n in ("dtype", "criterion", "ln_eps", "select_rule"):
             continue
         setattr(c, n, int(cfg[n] if n != "max_batch" else cfg.get("max_batch", cfg.get("batch"))))
     dt = cfg["dtype"]
@@ -148,6 +151,9 @@ def lazymar_create(cfg, weights):
     cr = cfg.get("criterion", "value")
     c.criterion = {"value": LAZYMAR_CRITERION_VALUE, "feature": LAZYMAR_CRITERION_FEATURE}.get(cr, cr)
     c.ln_eps = float(cfg.get("ln_eps", 1e-6))
+    sr = cfg.get("select_rule", LAZYMAR_SELECT_LEAST_SIMILAR)
+    c.select_rule = {"least_similar": LAZYMAR_SELECT_LEAST_SIMILAR, "most_similar": LAZYMAR_SELECT_MOST_SIMILAR,
+                     "random": LAZYMAR_SELECT_RANDOM}.get(sr, sr)
     keep = []
 
     def p(a):
@@ -172,8 +178,9 @@ def lazymar_create(cfg, weights):
     return Handle(h.value, c)
 
 
-def _step_in(latents, mask, labels, batch):
-    return lazymar_step_in(_ptr(latents), _ptr(mask), _ptr(labels), int(batch))
+def _step_in(latents, mask, labels, batch, select_priority=None, select_keys=None):
+    return lazymar_step_in(_ptr(latents), _ptr(mask), _ptr(labels), int(batch), _ptr(select_priority),
+                           _ptr(select_keys))
 
 
 def lazymar_full_step(h, latents, mask, labels, batch, gamma, z_out=None, guided_out=None, stream=None):
@@ -183,8 +190,8 @@ def lazymar_full_step(h, latents, mask, labels, batch, gamma, z_out=None, guided
 
 
 def lazymar_cached_step(h, latents, mask, labels, batch, n_compute, use_cond_cache, gamma, idx_in=None, idx_out=None,
-                        z_out=None, guided_out=None, stream=None):
-    si = _step_in(latents, mask, labels, batch)
+                        z_out=None, guided_out=None, stream=None, select_priority=None, select_keys=None):
+    si = _step_in(latents, mask, labels, batch, select_priority, select_keys)
     _check(lib().lazymar_cached_step(h.ptr, ctypes.byref(si), int(n_compute), int(bool(use_cond_cache)),
                                      float(gamma), _ptr(idx_in), _ptr(idx_out), _ptr(z_out), _ptr(guided_out),
                                      _stream(stream)))
@@ -193,6 +200,13 @@ def lazymar_cached_step(h, latents, mask, labels, batch, n_compute, use_cond_cac
 def lazymar_select_tokens(dtype, v_cur, v_cache, rows, T, D, n_compute, idx_out, stream=None):
     _check(lib().lazymar_select_tokens(int(dtype), _ptr(v_cur), _ptr(v_cache), int(rows), int(T), int(D),
                                        int(n_compute), _ptr(idx_out), _stream(stream)))
+
+
+def lazymar_select_tokens_ex(dtype, v_cur, v_cache, rows, T, D, n_compute, rule, priority, keys, idx_out,
+                             stream=None):
+    _check(lib().lazymar_select_tokens_ex(int(dtype), _ptr(v_cur), _ptr(v_cache), int(rows), int(T), int(D),
+                                          int(n_compute), int(rule), _ptr(priority), _ptr(keys), _ptr(idx_out),
+                                          _stream(stream)))
 
 
 def lazymar_select_tokens_noalloc(dtype, v_cur, v_cache, rows, T, D, n_compute, idx_out, stream=None):

@@ -64,7 +64,8 @@ def _cfg(**kw):
 
 @pytest.mark.parametrize("bad,status", [(dict(sel_layers=0), 1), (dict(sel_layers=3), 1), (dict(width=200), 6),
                                         (dict(width=384, heads=3), 6), (dict(heads=2, dtype="bf16"), 6),
-                                        (dict(token_dim=65), 6), (dict(max_batch=0), 1), (dict(dtype=7), 1)])
+                                        (dict(token_dim=65), 6), (dict(max_batch=0), 1), (dict(dtype=7), 1),
+                                        (dict(select_rule=3), 1)])
 def test_create_rejects_bad_configs_before_touching_the_device(lib, bad, status):
     with pytest.raises(lm.LazymarError) as e:
         _create_raw(lib, _cfg(**bad))
@@ -74,11 +75,12 @@ def test_create_rejects_bad_configs_before_touching_the_device(lib, bad, status)
 def _create_raw(lib, cfg):
     c = lm.lazymar_config()
     for n, _ in lm.lazymar_config._fields_:
-        if n not in ("dtype", "criterion", "ln_eps"):
+        if n not in ("dtype", "criterion", "ln_eps", "select_rule"):
             setattr(c, n, cfg[n])
     c.dtype = {"fp32": 0, "bf16": 1}.get(cfg["dtype"], cfg["dtype"])
     c.criterion = 0
     c.ln_eps = 1e-6
+    c.select_rule = cfg.get("select_rule", 0)
     w = lm.lazymar_weights()
     blocks = (lm.lazymar_block_weights * 1)()
     w.blocks = blocks
@@ -112,6 +114,8 @@ def test_component_argument_checks(lib):
     assert lib.lazymar_select_tokens(1, None, None, 2, 10, 12, 3, None, None) == 1      # D % 8
     assert lib.lazymar_select_tokens(1, None, None, 2, 10, 16, 11, None, None) == 1     # N > T
     assert lib.lazymar_select_tokens(5, None, None, 2, 10, 16, 3, None, None) == 1      # dtype
+    assert lib.lazymar_select_tokens_ex(1, None, None, 2, 10, 16, 3, 3, None, None, None, None) == 1  # rule
+    assert lib.lazymar_select_tokens_ex(1, None, None, 2, 10, 16, 11, 0, None, None, None, None) == 1  # N > T
     assert lib.lazymar_cfg_combine(1, 3, None, None, None, 1.0, 8, None, None, None) == 1
     assert lib.lazymar_attention(1, None, None, None, None, 1, 1, 1, 2, 96, None) == 6  # head width 96
     assert lib.lazymar_layernorm(1, None, None, None, None, None, 4, 200, 1e-6, None) == 6

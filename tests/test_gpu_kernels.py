@@ -42,6 +42,40 @@ def test_select_tokens_bit_exact(rows, T, D, N, dtype):
     assert torch.equal(g_ref, g_cur)
 
 
+@pytest.mark.parametrize("rule", [lm.LAZYMAR_SELECT_LEAST_SIMILAR, lm.LAZYMAR_SELECT_MOST_SIMILAR,
+                                  lm.LAZYMAR_SELECT_RANDOM])
+@pytest.mark.parametrize("with_prio", [False, True])
+@pytest.mark.parametrize("rows,T,D,N,dtype", [
+    (64, 320, 768, 50, "bf16"),    # MAR-B
+    (2, 80, 256, 20, "fp32"),      # tiny
+    (5, 100, 16, 37, "bf16"),
+    (3, 320, 768, 320, "bf16"),    # N = T
+    (4, 513, 64, 129, "fp32"),
+])
+def test_select_rules_bit_exact(rule, with_prio, rows, T, D, N, dtype):
+    """Selection strategies of Table 3 (V, IV, III) with and without priority
+    classes (observation-based / type strategies) against the oracle on the
+    same buffers: indices bit-exact, reference updated."""
+    torch = torch_cuda()
+    cur, ref = synth.similarity_inputs(rows, T, D, seed=rows * 1000 + T + rule, dtype=dtype)
+    rng = np.random.default_rng(rows + T + 7 * rule + with_prio)
+    prio = rng.integers(0, 3, size=(rows, T)).astype(np.uint8) if with_prio else None
+    keys = rng.integers(0, 1 << 32, size=(rows, T), dtype=np.uint64).astype(np.uint32)
+    keys[:, 1::7] = keys[:, 0:1]  # repeated keys: the index decides
+    g_cur, g_ref = dev(cur, dtype), dev(ref, dtype)
+    g_prio = torch.from_numpy(prio).cuda() if with_prio else None
+    g_keys = torch.from_numpy(keys.view(np.int32)).cuda()
+    idx = torch.full((rows, max(N, 1)), -1, dtype=torch.int32, device="cuda")
+    lm.lazymar_select_tokens_ex(DT[dtype], g_cur, g_ref, rows, T, D, N, rule, g_prio, g_keys, idx)
+    sync()
+    got = idx.cpu().numpy()[:, :N]
+    for r in range(rows):
+        expect = O.select_by_rule(O.cosine_similarity(cur[r], ref[r]), N, rule,
+                                  None if prio is None else prio[r], keys[r])
+        assert got[r].tolist() == expect.tolist(), "row %d" % r
+    assert torch.equal(g_ref, g_cur)
+
+
 def _selection_edge_inputs(T, D, seed):
     """bf16 rows that exercise both similarity paths of the kernel.
 

@@ -55,14 +55,15 @@ class Run:
         lm.lazymar_sync(self.h)
         return host(z), host(g)
 
-    def cached(self, st, n, reuse, idx_in=None):
+    def cached(self, st, n, reuse, idx_in=None, priority=None, keys=None):
         lat, m = st
         z, g = self.outs()
         rows = self.B if reuse else 2 * self.B
         idx = self.torch.full((rows, max(n, 1)), -1, dtype=self.torch.int32, device="cuda")
         lm.lazymar_cached_step(self.h, dev(lat), dev_int(m), dev_int(self.labels), self.B, n, reuse, GAMMA,
                                None if idx_in is None else dev_int(np.ascontiguousarray(idx_in, np.int32)), idx, z,
-                               g)
+                               g, select_priority=None if priority is None else dev_int(priority),
+                               select_keys=None if keys is None else dev_int(keys.view(np.int32)))
         lm.lazymar_sync(self.h)
         return host(z), host(g), idx.cpu().numpy()[:, :n]
 
@@ -101,6 +102,70 @@ def test_tiny_full_then_cached_step(tiny):
     for row in range(2):
         keep = [t - nb for t in range(nb, cfg["T"]) if t not in set(I1g[row].tolist())]
         assert np.array_equal(z1g[row, keep], z0g[row, keep])
+
+
+def _valid_rule_selection(I, S, n, rule, prio, keys, margin=1e-6):
+    """I is a valid choice of the n first tokens under the rule's order, with
+    similarities allowed to differ from the oracle's S by `margin` (fp32)."""
+    I = list(I)
+    if len(I) != n or I != sorted(set(I)):
+        return False
+    rest = [t for t in range(len(S)) if t not in set(I)]
+    for a in I:
+        for b in rest:
+            if prio is not None and prio[a] != prio[b]:
+                if prio[a] < prio[b]:
+                    return False
+                continue
+            if rule == lm.LAZYMAR_SELECT_RANDOM:
+                if (int(keys[b]), b) < (int(keys[a]), a):
+                    return False
+            elif rule == lm.LAZYMAR_SELECT_LEAST_SIMILAR:
+                if S[b] < S[a] - margin:
+                    return False
+            elif S[b] > S[a] + margin:
+                return False
+    return True
+
+
+@pytest.mark.parametrize("rule", [lm.LAZYMAR_SELECT_LEAST_SIMILAR, lm.LAZYMAR_SELECT_MOST_SIMILAR,
+                                  lm.LAZYMAR_SELECT_RANDOM])
+@pytest.mark.parametrize("with_prio", [False, True])
+def test_tiny_cached_step_selection_rules(rule, with_prio):
+    """A cached step under each selection strategy of Table 3. Priority 1 marks
+    the image tokens decoded since the last step (the observation-based
+    strategy); the random keys are seeded inputs. The GPU's selection must be a
+    valid prefix of the rule's order under the oracle's similarities (exact
+    for priorities and keys). Features match the oracle run on that selection."""
+    r = Run("tiny", select_rule=rule)
+    cfg = r.cfg
+    (lat0, m0), (lat1, m1) = synth.tiny_state(cfg, r.order, r.table)
+    N, T, nb = synth.n_compute(cfg), cfg["T"], cfg["n_buffer"]
+    rows = 2 * r.B
+    prio = None
+    if with_prio:
+        decoded_now = (np.asarray(m0) != 0) & (np.asarray(m1) == 0)            # [B, n_img]
+        p = np.zeros((r.B, T), np.uint8)
+        p[:, nb:] = decoded_now
+        prio = np.ascontiguousarray(np.concatenate([p, p], axis=0))           # both pathways
+    keys = np.random.default_rng(5).integers(0, 1 << 32, size=(rows, T), dtype=np.uint64).astype(np.uint32)
+    c = O.Cache(cfg, 1)
+    O.full_step(cfg, r.W, c, lat0, m0, r.labels, GAMMA)
+    _, _, I_or, S_or = O.cached_step(cfg, r.W, c, lat1, m1, r.labels, N, False, GAMMA, rule=rule, priority=prio,
+                                     keys=keys)
+    r.full((lat0, m0))
+    z1g, g1g, I1g = r.cached((lat1, m1), N, False, priority=prio,
+                             keys=keys if rule == lm.LAZYMAR_SELECT_RANDOM else None)
+    for row in range(rows):
+        assert _valid_rule_selection(I1g[row], S_or[row], N, rule, None if prio is None else prio[row], keys[row])
+    if rule == lm.LAZYMAR_SELECT_RANDOM:
+        assert I1g.tolist() == I_or.tolist()
+    # features: the oracle on the GPU's selection
+    c2 = O.Cache(cfg, 1)
+    O.full_step(cfg, r.W, c2, lat0, m0, r.labels, GAMMA)
+    z1, g1, _, _ = O.cached_step(cfg, r.W, c2, lat1, m1, r.labels, N, False, GAMMA, idx=I1g)
+    assert max_rel(z1g, z1) < TOL["fp32"] and max_rel(g1g, g1) < TOL["fp32"]
+    r.h.close()
 
 
 def test_tiny_full_ratio_cached_step_equals_full_step(tiny):

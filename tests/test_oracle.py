@@ -229,6 +229,69 @@ def test_select_picks_least_similar_and_nan_first():
     assert list(O.select_compute(S, 4)) == [1, 3, 4, 5]
 
 
+def _rule_precedes(a, b, S, rule, prio, keys):
+    """Token a is taken before token b under a selection rule of Table 3,
+    written as explicit comparisons (priority, then the rule, then index)."""
+    pa, pb = (prio[a], prio[b]) if prio is not None else (0, 0)
+    if pa != pb:
+        return pa > pb
+    if rule == O.SELECT_RANDOM:
+        ka, kb = int(keys[a]), int(keys[b])
+    else:
+        sa = -math.inf if math.isnan(S[a]) else S[a]
+        sb = -math.inf if math.isnan(S[b]) else S[b]
+        ka, kb = (sa, sb) if rule == O.SELECT_LEAST_SIMILAR else (-sa, -sb)
+    if ka != kb:
+        return ka < kb
+    return a < b
+
+
+@pytest.mark.parametrize("rule", [O.SELECT_LEAST_SIMILAR, O.SELECT_MOST_SIMILAR, O.SELECT_RANDOM])
+@pytest.mark.parametrize("with_prio", [False, True])
+@pytest.mark.parametrize("T,n", [(1, 0), (1, 1), (9, 4), (16, 7), (16, 16)])
+def test_select_by_rule_is_a_prefix_of_the_order(rule, with_prio, T, n):
+    """Every selected token precedes every unselected one under the stated
+    order, the set has n members, ascending; ties in S, -0/+0 and NaN included."""
+    rng = np.random.default_rng(T * 31 + n + rule * 7 + with_prio)
+    S = np.round(rng.standard_normal(T), 1)  # rounding makes ties
+    if T > 3:
+        S[1] = np.nan
+        S[2], S[3] = 0.0, -0.0
+    prio = rng.integers(0, 2, T) if with_prio else None
+    keys = rng.integers(0, 6, T).astype(np.uint32)  # repeated keys: ties
+    got = list(O.select_by_rule(S, n, rule, prio, keys))
+    assert len(got) == n and got == sorted(got)
+    rest = [t for t in range(T) if t not in got]
+    for a in got:
+        for b in rest:
+            assert _rule_precedes(a, b, S, rule, prio, keys), (a, b)
+
+
+def test_select_by_rule_worked_cases():
+    """Hand-worked six-token row (Table 3 strategies; priority 1 marks tokens
+    that must be recomputed, as the observation-based strategy does for
+    tokens decoded at steps t-1 and t)."""
+    S = np.array([0.9, 0.1, np.nan, 0.5, 0.1, -0.2])
+    prio = np.array([0, 0, 0, 1, 0, 1])
+    keys = np.array([5, 3, 9, 1, 0, 2], np.uint32)
+    # strategy V: least similar first; NaN counts as -inf
+    assert list(O.select_by_rule(S, 3)) == [1, 2, 5]
+    # strategy IV: most similar first; the NaN token comes last
+    assert list(O.select_by_rule(S, 3, O.SELECT_MOST_SIMILAR)) == [0, 1, 3]
+    # strategy III: ascending random keys
+    assert list(O.select_by_rule(S, 3, O.SELECT_RANDOM, keys=keys)) == [3, 4, 5]
+    # priority first (tokens 3 and 5), then each rule fills the remaining slot
+    assert list(O.select_by_rule(S, 3, O.SELECT_LEAST_SIMILAR, prio)) == [2, 3, 5]
+    assert list(O.select_by_rule(S, 3, O.SELECT_MOST_SIMILAR, prio)) == [0, 3, 5]
+    assert list(O.select_by_rule(S, 3, O.SELECT_RANDOM, prio, keys)) == [3, 4, 5]
+    # more priority tokens than the budget: the rule orders them
+    assert list(O.select_by_rule(S, 1, O.SELECT_LEAST_SIMILAR, prio)) == [5]
+    assert list(O.select_by_rule(S, 1, O.SELECT_MOST_SIMILAR, prio)) == [3]
+    # without priority, the default rule is select_compute
+    for n in range(7):
+        assert list(O.select_by_rule(S, n)) == list(O.select_compute(S, n))
+
+
 def test_selection_recomputes_the_changed_tokens():
     # Strategy V (Table 3): the tokens whose representation moved most since the
     # last step are recomputed.
