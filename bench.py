@@ -107,6 +107,29 @@ def selection_inputs(cfg, masks, rule_name, seed_offset):
     return prio, None
 
 
+def rank_seed_offset(rank):
+    """Seed offset of a rank's inputs: every rank decodes its own batch of pairs
+    (weak scaling; pairs are independent, so no data-path collective)."""
+    return rank * 101
+
+
+def max_over_ranks(values, device):
+    """Element-wise maximum over all ranks (the slowest rank's timing)."""
+    import torch
+    import torch.distributed as dist
+    if not dist.is_initialized() or dist.get_world_size() == 1:
+        return [float(v) for v in values]
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t]
+
+
+def job_images_per_s(world, batch, decodes, ms):
+    """Whole-job throughput: `world` ranks each decode `batch` pairs `decodes`
+    times within `ms` (the maximum over ranks)."""
+    return world * batch * decodes / (ms / 1000.0)
+
+
 def decode_inputs(cfg, seed_offset):
     """Latents and masks of every decoding step for one batch (numpy)."""
     order = synth.make_order(cfg, seed=2 + seed_offset)
@@ -266,11 +289,11 @@ def run_ours(args, cfg):
     B, N, steps = cfg["batch"], synth.n_compute(cfg), cfg["steps"]
     W = synth.make_weights(cfg)
     h = lm.lazymar_create(dict(cfg, max_batch=B, select_rule=SELECT_RULES[args.select]), W)
-    lat_np, mask_np, labels_np = decode_inputs(cfg, rank * 101)
+    lat_np, mask_np, labels_np = decode_inputs(cfg, rank_seed_offset(rank))
     lat = torch.from_numpy(lat_np).cuda()
     mask = torch.from_numpy(mask_np).cuda()
     labels = torch.from_numpy(labels_np).cuda()
-    prio_np, keys_np = selection_inputs(cfg, mask_np, args.select, rank * 101)
+    prio_np, keys_np = selection_inputs(cfg, mask_np, args.select, rank_seed_offset(rank))
     prio = None if prio_np is None else torch.from_numpy(prio_np).cuda()
     keys = None if keys_np is None else torch.from_numpy(keys_np.view(np.int32)).cuda()
     guided = torch.empty((B, cfg["n_img"], cfg["width"]), dtype=torch.bfloat16, device="cuda")
@@ -310,9 +333,8 @@ def run_ours(args, cfg):
         wall = time.perf_counter() - t0
         ms = e0.elapsed_time(e1)
         if world > 1:
-            t = torch.tensor([ms, wall * 1000.0], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms, wall = float(t[0]), float(t[1]) / 1000.0
+            ms, wall_ms = max_over_ranks([ms, wall * 1000.0], "cuda")
+            wall = wall_ms / 1000.0
             dist.barrier()
         return ms, wall
 
@@ -328,7 +350,7 @@ def run_ours(args, cfg):
     launches = sum(v["launches"] for v in st.values())
     lm.lazymar_sync(h, stream)
     ms_per_step = ms / args.steps
-    images_per_s = world * B * args.steps / (ms / 1000.0)
+    images_per_s = job_images_per_s(world, B, args.steps, ms)
 
     # 2) per-kernel device time: events around every launch (separate pass)
     lm.lazymar_reset_stats(h)
@@ -350,7 +372,7 @@ def run_ours(args, cfg):
     for _ in range(1):
         decode(full_only=True)
     ms_full, _ = timed(lambda: decode(full_only=True), args.steps)
-    full_images_per_s = world * B * args.steps / (ms_full / 1000.0)
+    full_images_per_s = job_images_per_s(world, B, args.steps, ms_full)
 
     # 4) end to end through the C ABI with host buffers (pinned), copies inside
     host = {"lat": lat.cpu().pin_memory(), "mask": mask.cpu().pin_memory(), "labels": labels.cpu().pin_memory(),
@@ -359,7 +381,7 @@ def run_ours(args, cfg):
             "keys": None if keys is None else keys.cpu().pin_memory()}
     decode(host=host)
     ms_e2e, _ = timed(lambda: decode(host=host), args.steps)
-    e2e_images_per_s = world * B * args.steps / (ms_e2e / 1000.0)
+    e2e_images_per_s = job_images_per_s(world, B, args.steps, ms_e2e)
     # selection inputs are copied on cached steps only, for the rows they run
     cached_rows = sum(0 if f else (B if r else 2 * B) for f, r in plan)
     sel_bytes = cached_rows * cfg["T"] * ((1 if prio is not None else 0) + (4 if keys is not None else 0))

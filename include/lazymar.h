@@ -294,6 +294,15 @@ lazymar_status lazymar_sync(lazymar_handle *h, void *stream);
 /* As lazymar_sync for the component entry points of the current device. */
 lazymar_status lazymar_device_check(void *stream);
 
+/* Failure-detection self-test (no counterpart in the paper): launches one CTA
+ * that waits on an mbarrier nothing completes, with a wait limit of limit_us
+ * microseconds (1..1000000), the same bounded wait every pipelined kernel
+ * uses. The wait runs out, the kernel raises LAZYMAR_ERR_TIMEOUT in the
+ * component error word and returns; the next lazymar_device_check on the
+ * stream reports LAZYMAR_ERR_TIMEOUT (and clears it), and the device stays
+ * usable. Returns INVALID_ARG outside the limit range. */
+lazymar_status lazymar_selftest_wait(int limit_us, void *stream);
+
 /* Per kernel class: launches, algorithmic flops and bytes, and (while
  * profiling is on) device time from CUDA events recorded around each launch on
  * its stream. lazymar_get_stats waits for the recorded events. */

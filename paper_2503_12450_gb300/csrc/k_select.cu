@@ -418,3 +418,31 @@ extern "C" lazymar_status lazymar_select_tokens_noalloc(int dtype, const void* v
   return LAZYMAR_OK;
 }
 
+namespace lm {
+
+// ---------------------------------------------------------------------------
+// Bounded-wait diagnostic
+// ---------------------------------------------------------------------------
+// Every pipelined kernel waits on mbarriers with a time limit: on expiry it
+// raises its abort flag and ERR_TIMEOUT in the device error word, stops, and
+// returns normally, so the context stays usable and the host learns of the
+// failure from lazymar_sync / lazymar_device_check. This kernel drives that
+// path on purpose: its barrier expects one arrival that never comes.
+__global__ void stuck_wait_kernel(unsigned* err, unsigned long long limit_ns) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  mbar_wait_limit(&bar, 0, &abort_flag, err, limit_ns);
+}
+
+cudaError_t launch_stuck_wait(const Ctx& c, uint64_t limit_ns) {
+  stuck_wait_kernel<<<1, 32, 0, c.stream>>>(c.err, (unsigned long long)limit_ns);
+  return cudaGetLastError();
+}
+
+}  // namespace lm

@@ -811,6 +811,14 @@ extern "C" lazymar_status lazymar_sync(lazymar_handle* h, void* stream) {
   return read_error_word(h->err, static_cast<cudaStream_t>(stream));
 }
 
+extern "C" lazymar_status lazymar_selftest_wait(int limit_us, void* stream) {
+  if (limit_us < 1 || limit_us > 1000000) return fail(LAZYMAR_ERR_INVALID_ARG, "limit_us outside 1..1000000");
+  Ctx c;
+  LM_TRY(component_ctx(stream, &c));
+  cudaError_t e = launch_stuck_wait(c, (uint64_t)limit_us * 1000ull);
+  return e == cudaSuccess ? LAZYMAR_OK : cuda_fail(e, "stuck-wait kernel");
+}
+
 extern "C" lazymar_status lazymar_device_check(void* stream) {
   Ctx c;
   LM_TRY(component_ctx(stream, &c));

@@ -204,21 +204,25 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // Waits for the phase with the given parity to complete. Gives up (returns
 // false) when *abort_flag is raised by another thread of the CTA or after
 // kWaitLimitNs, in which case it raises *abort_flag and ERR_TIMEOUT.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                          unsigned* err) {
+__device__ __forceinline__ bool mbar_wait_limit(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                                unsigned* err, uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((i & 63u) == 0) {
       if (*abort_flag) return false;
-      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      if (globaltimer_ns() - t0 > limit_ns) {
         *abort_flag = 1;
         atomicOr(err, ERR_TIMEOUT);
         return false;
       }
     }
   }
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                          unsigned* err) {
+  return mbar_wait_limit(bar, parity, abort_flag, err, kWaitLimitNs);
 }
 // Orders this thread's view of prior generic-proxy shared-memory accesses
 // (made visible to it by a CTA barrier) before its subsequent async-proxy
@@ -388,6 +392,9 @@ cudaError_t launch_cast(const Ctx& c, int dtype, const float* x, void* y, size_t
 
 cudaError_t launch_similarity(const Ctx& c, int dtype, const void* cur, void* cache, double* S, int rows, int T,
                               int D, bool copy);
+// Diagnostic: one CTA waits on an mbarrier that nothing completes, for at most
+// limit_ns (the bounded-wait failure path of every pipelined kernel).
+cudaError_t launch_stuck_wait(const Ctx& c, uint64_t limit_ns);
 cudaError_t launch_topk(const Ctx& c, const double* S, int rows, int T, int N, int* idx, int* row_map,
                         int rule = 0, const uint8_t* prio = nullptr, const uint32_t* keys = nullptr);
 cudaError_t launch_idx_check(const Ctx& c, const int* idx_in, int rows, int T, int N, int* idx, int* row_map);

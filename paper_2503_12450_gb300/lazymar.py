@@ -89,6 +89,7 @@ def lib():
         "lazymar_plan_step": (i, [i, i, i, i, i]),
         "lazymar_sync": (st, [vp, vp]),
         "lazymar_device_check": (st, [vp]),
+        "lazymar_selftest_wait": (st, [i, vp]),
         "lazymar_set_profiling": (st, [vp, i]),
         "lazymar_set_graphs": (st, [vp, i]),
         "lazymar_get_stats": (st, [vp, ctypes.POINTER(lazymar_stats)]),
@@ -247,6 +248,10 @@ def lazymar_plan_step(k, k0, tau, tau_cfg, use_cond_cache=True):
 
 def lazymar_sync(h, stream=None):
     _check(lib().lazymar_sync(h.ptr, _stream(stream)))
+
+
+def lazymar_selftest_wait(limit_us, stream=None):
+    _check(lib().lazymar_selftest_wait(int(limit_us), _stream(stream)))
 
 
 def lazymar_device_check(stream=None):

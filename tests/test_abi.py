@@ -115,6 +115,7 @@ def test_component_argument_checks(lib):
     assert lib.lazymar_select_tokens(1, None, None, 2, 10, 16, 11, None, None) == 1     # N > T
     assert lib.lazymar_select_tokens(5, None, None, 2, 10, 16, 3, None, None) == 1      # dtype
     assert lib.lazymar_select_tokens_ex(1, None, None, 2, 10, 16, 3, 3, None, None, None, None) == 1  # rule
+    assert lib.lazymar_selftest_wait(0, None) == 1                                      # limit
     assert lib.lazymar_select_tokens_ex(1, None, None, 2, 10, 16, 11, 0, None, None, None, None) == 1  # N > T
     assert lib.lazymar_cfg_combine(1, 3, None, None, None, 1.0, 8, None, None, None) == 1
     assert lib.lazymar_attention(1, None, None, None, None, 1, 1, 1, 2, 96, None) == 6  # head width 96

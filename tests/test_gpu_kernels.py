@@ -285,3 +285,25 @@ def test_gelu_epilogue_matches_erf_gelu():
     sync()
     err = np.abs(host(out) - O.gelu(x.astype(np.float64)))
     assert (err <= 1e-6 * np.maximum(1.0, np.abs(x))).all(), float(err.max())
+
+
+# --------------------------------------------------------------------------
+# Failure detection: a bounded device wait that runs out
+# --------------------------------------------------------------------------
+
+def test_bounded_wait_expires_and_device_stays_usable():
+    """The self-test kernel waits 50 ms on an mbarrier nothing completes: the
+    wait gives up, the host reads LAZYMAR_ERR_TIMEOUT (then the word is clear),
+    and kernels launched afterwards still run correctly."""
+    import time
+    lm.lazymar_device_check()
+    t0 = time.perf_counter()
+    lm.lazymar_selftest_wait(50000)
+    with pytest.raises(lm.LazymarError) as e:
+        lm.lazymar_device_check()
+    assert e.value.status == 5                       # LAZYMAR_ERR_TIMEOUT
+    assert time.perf_counter() - t0 < 10
+    lm.lazymar_device_check()                        # reported once, then clear
+    _linear_case("bf16", lm.LAZYMAR_EPI_BIAS, 200, 256, 128, 1, seed=5)
+    lm.lazymar_device_check()
+
