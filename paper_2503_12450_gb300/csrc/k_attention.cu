@@ -437,12 +437,19 @@ __global__ void __launch_bounds__(at2::THREADS, 3) attention_tc_kernel(const __g
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars[B_S_FREE]);
+      // row max of the raw scores; keys beyond T (the last chunk only) drop out
       float mloc = -FLT_MAX;
+      if (c * KC + KC <= T) {
 #pragma unroll
-      for (int i = 0; i < 64; ++i) {
-        sv[i] = (c * KC + i < T) ? sv[i] * scale_log2 : -FLT_MAX;
-        mloc = fmaxf(mloc, sv[i]);
+        for (int i = 0; i < 64; ++i) mloc = fmaxf(mloc, sv[i]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 64; ++i) {
+          sv[i] = (c * KC + i < T) ? sv[i] : -FLT_MAX;
+          mloc = fmaxf(mloc, sv[i]);
+        }
       }
+      mloc *= scale_log2;  // log2 units (scale_log2 > 0 keeps the maximum)
       float alpha = 1.f;
       bool raise = false;
       if (c == 0) {
@@ -456,7 +463,8 @@ __global__ void __launch_bounds__(at2::THREADS, 3) attention_tc_kernel(const __g
       uint32_t pk[32];
 #pragma unroll
       for (int i = 0; i < 32; ++i) {
-        const float p0 = exp2_approx(sv[2 * i] - m_run), p1 = exp2_approx(sv[2 * i + 1] - m_run);
+        const float p0 = exp2_approx(fmaf(sv[2 * i], scale_log2, -m_run)),
+                    p1 = exp2_approx(fmaf(sv[2 * i + 1], scale_log2, -m_run));
         psum += p0 + p1;
         pk[i] = pack_bf16(p0, p1);
       }
