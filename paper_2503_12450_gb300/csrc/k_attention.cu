@@ -441,7 +441,7 @@ __global__ void __launch_bounds__(at2::THREADS, 3) attention_tc_kernel(const __g
       float mloc = -FLT_MAX;
       if (c * KC + KC <= T) {
 #pragma unroll
-        for (int i = 0; i < 64; ++i) mloc = fmaxf(mloc, sv[i]);
+        for (int i = 0; i < 64; i += 2) mloc = fmax3(mloc, sv[i], sv[i + 1]);
       } else {
 #pragma unroll
         for (int i = 0; i < 64; ++i) {
@@ -459,15 +459,22 @@ __global__ void __launch_bounds__(at2::THREADS, 3) attention_tc_kernel(const __g
         alpha = exp2_approx(m_run - mloc);
         m_run = mloc;
       }
-      float psum = 0.f;
+      // exponent arguments and the row sum two keys per instruction (the
+      // softmax is bound by instruction issue)
+      const unsigned long long sc2 = f32x2_pack(scale_log2, scale_log2), nm2 = f32x2_pack(-m_run, -m_run);
+      unsigned long long ps2 = f32x2_pack(0.f, 0.f);
       uint32_t pk[32];
 #pragma unroll
       for (int i = 0; i < 32; ++i) {
-        const float p0 = exp2_approx(fmaf(sv[2 * i], scale_log2, -m_run)),
-                    p1 = exp2_approx(fmaf(sv[2 * i + 1], scale_log2, -m_run));
-        psum += p0 + p1;
+        float x0, x1;
+        f32x2_unpack(f32x2_fma(f32x2_pack(sv[2 * i], sv[2 * i + 1]), sc2, nm2), x0, x1);
+        const float p0 = exp2_approx(x0), p1 = exp2_approx(x1);
+        ps2 = f32x2_add(ps2, f32x2_pack(p0, p1));
         pk[i] = pack_bf16(p0, p1);
       }
+      float ps0, ps1;
+      f32x2_unpack(ps2, ps0, ps1);
+      const float psum = ps0 + ps1;
       // PV(c-1) must be complete before O is rescaled or P is overwritten.
       if (c > 0) {
         ok = __all_sync(0xffffffffu, mbar_wait(&bars[B_O_DONE], (uint32_t)(c - 1) & 1u, abort_flag, err));
