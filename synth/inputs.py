@@ -208,3 +208,60 @@ def distinct_rows(n, total, seed):
     """n distinct row indices out of `total`, in random order (a scatter map)."""
     rng = np.random.Generator(np.random.PCG64(seed))
     return rng.permutation(total)[:n].astype(np.int32)
+
+
+# ----------------------------------------------------------------------------
+# Diffusion head (the per-token denoiser that draws each decoded token's latent)
+# ----------------------------------------------------------------------------
+# Width and depth follow the MAR head sizes that go with the transformer
+# configurations; n_steps sampling steps over n_train training steps.
+HEAD_CONFIGS = {
+    "tiny": dict(width=128, depth=2, freq_dim=256, n_train=1000, n_steps=10),
+    "mar_b": dict(width=1024, depth=6, freq_dim=256, n_train=1000, n_steps=100),
+    "mar_l": dict(width=1280, depth=8, freq_dim=256, n_train=1000, n_steps=100),
+    "mar_h": dict(width=1536, depth=12, freq_dim=256, n_train=1000, n_steps=100),
+}
+
+
+def head_config(name, **overrides):
+    c = dict(HEAD_CONFIGS[name])
+    c.update(overrides)
+    c["name"] = name
+    return c
+
+
+def make_head_weights(hc, cond_dim, token_dim, seed=4, bf16=True):
+    """Random-init head weights ([out, in] layout), N(0, 0.02) throughout."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    w, f = hc["width"], hc["freq_dim"]
+    W = {
+        "t_w1": _normal(rng, (w, f), 0.02), "t_b1": _normal(rng, (w,), 0.02),
+        "t_w2": _normal(rng, (w, w), 0.02), "t_b2": _normal(rng, (w,), 0.02),
+        "c_w": _normal(rng, (w, cond_dim), 0.02), "c_b": _normal(rng, (w,), 0.02),
+        "in_w": _normal(rng, (w, token_dim), 0.02), "in_b": _normal(rng, (w,), 0.02),
+        "blocks": [],
+    }
+    for _ in range(hc["depth"]):
+        W["blocks"].append({
+            "ada_w": _normal(rng, (3 * w, w), 0.02), "ada_b": _normal(rng, (3 * w,), 0.02),
+            "w1": _normal(rng, (w, w), 0.02), "b1": _normal(rng, (w,), 0.02),
+            "w2": _normal(rng, (w, w), 0.02), "b2": _normal(rng, (w,), 0.02),
+        })
+    W["f_ada_w"] = _normal(rng, (2 * w, w), 0.02)
+    W["f_ada_b"] = _normal(rng, (2 * w,), 0.02)
+    W["out_w"] = _normal(rng, (2 * token_dim, w), 0.02)
+    W["out_b"] = _normal(rng, (2 * token_dim,), 0.02)
+    if bf16:
+        for k in list(W):
+            if k != "blocks":
+                W[k] = round_bf16(W[k])
+        for b in W["blocks"]:
+            for k in b:
+                b[k] = round_bf16(b[k])
+    return W
+
+
+def make_head_noise(n_steps, M, token_dim, seed=5):
+    """noise[0] = starting latents, noise[i] = noise added after denoising step i."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    return rng.standard_normal((n_steps, M, token_dim), dtype=np.float32)
