@@ -297,10 +297,12 @@ def run_ours(args, cfg):
     prio = None if prio_np is None else torch.from_numpy(prio_np).cuda()
     keys = None if keys_np is None else torch.from_numpy(keys_np.view(np.int32)).cuda()
     guided = torch.empty((B, cfg["n_img"], cfg["width"]), dtype=torch.bfloat16, device="cuda")
+    zbuf = torch.empty((2 * B, cfg["n_img"], cfg["width"]), device="cuda",
+                       dtype=torch.bfloat16 if cfg["dtype"] == "bf16" else torch.float32)
     stream = torch.cuda.current_stream()
     dev_in = {"lat": lat, "mask": mask, "labels": labels, "guided": guided, "prio": prio, "keys": keys}
 
-    def decode(full_only=False, host=None, step_events=None):
+    def decode(full_only=False, host=None, step_events=None, head_step=None):
         for k in range(steps):
             full, reuse = plan[k]
             src = host if host is not None else dev_in
@@ -309,11 +311,14 @@ def run_ours(args, cfg):
             r_k = None if src["keys"] is None else src["keys"][k]
             if step_events is not None:
                 step_events[k][0].record(stream)
+            z = None if head_step is None else zbuf
             if full or full_only:
-                lm.lazymar_full_step(h, l_k, m_k, lab, B, GAMMA, None, g, stream)
+                lm.lazymar_full_step(h, l_k, m_k, lab, B, GAMMA, z, g, stream)
             else:
-                lm.lazymar_cached_step(h, l_k, m_k, lab, B, N, reuse, GAMMA, None, None, None, g, stream,
+                lm.lazymar_cached_step(h, l_k, m_k, lab, B, N, reuse, GAMMA, None, None, z, g, stream,
                                        select_priority=p_k, select_keys=r_k)
+            if head_step is not None:
+                head_step(k)
             if step_events is not None:
                 step_events[k][1].record(stream)
         if host is not None:
@@ -389,6 +394,14 @@ def run_ours(args, cfg):
     d2h = steps * guided.numel() * 2
     lm.lazymar_sync(h, stream)
 
+    # 5) the whole MAR sampling step: after every decoding step the diffusion
+    # head draws the latents of the tokens that step decodes (100 denoising
+    # steps, guidance on the noise prediction)
+    with_head = None
+    if not args.no_head:
+        with_head = run_head_phase(args, cfg, lm, torch, mask_np, rank, stream, decode, timed, world, zbuf)
+    lm.lazymar_sync(h, stream)
+
     if rank != 0:
         h.close()
         dist.destroy_process_group()
@@ -430,6 +443,7 @@ def run_ours(args, cfg):
                 "d2h_bytes_per_step": int(d2h)},
         "gpu_launches": int(launches),
         "clocks": clocks.summary(),
+        "with_head": with_head,
         "wall_s": wall,
     }
     if not args.no_cpu_baseline and world == 1:
@@ -483,6 +497,66 @@ def profile_case(args, cfg):
     print(json.dumps({"profile_case": args.profile_case, "config": cfg["name"], "ok": True}), flush=True)
 
 
+HEAD_FOR = {"tiny": "tiny", "mar_b": "mar_b", "mar_l": "mar_l", "mar_h": "mar_h", "hires": "mar_l"}
+
+
+def decoded_positions(mask_np):
+    """Per decoding step, the image positions each pair decodes at that step
+    ([B, n_new]; masked at step k and known at step k + 1, all remaining ones at
+    the last step). The cosine schedule decodes the same count in every pair."""
+    steps = mask_np.shape[0]
+    out = []
+    for k in range(steps):
+        new = mask_np[k].astype(bool) & (~mask_np[k + 1].astype(bool) if k + 1 < steps else True)
+        counts = new.sum(axis=1)
+        assert np.all(counts == counts[0]), "pairs decode different token counts"
+        out.append(np.stack([np.flatnonzero(r) for r in new]).astype(np.int32) if counts[0] else None)
+    return out
+
+
+def run_head_phase(args, cfg, lm, torch, mask_np, rank, stream, decode, timed, world, zbuf):
+    """Decodes with the diffusion head after every step; returns the report
+    (images/s of whole MAR sampling, head time and launches), or None."""
+    B, n_img, D, td = cfg["batch"], cfg["n_img"], cfg["width"], cfg["token_dim"]
+    hc = synth.head_config(HEAD_FOR[cfg["name"]])
+    pos = decoded_positions(mask_np)
+    max_new = max(p.shape[1] for p in pos if p is not None)
+    HW = synth.make_head_weights(hc, D, td, seed=4 + rank_seed_offset(rank))
+    hd = lm.lazymar_head_create(hc, D, td, HW, max_tokens=B * max_new, z_dtype=cfg["dtype"])
+    pos_d = [None if p is None else torch.from_numpy(p).cuda() for p in pos]
+    noise_d = [None if p is None else torch.from_numpy(synth.make_head_noise(hc["n_steps"], B * p.shape[1], td,
+                                                                              seed=100 + k + rank_seed_offset(rank))).cuda()
+               for k, p in enumerate(pos)]
+    x_d = [None if p is None else torch.empty((B * p.shape[1], td), device="cuda") for p in pos]
+
+    def head_step(k):
+        # zbuf holds step k's features of both pathways (the step's z output)
+        if pos_d[k] is not None:
+            lm.lazymar_head_sample(hd, zbuf, B, n_img, pos_d[k], pos_d[k].shape[1], noise_d[k], GAMMA, 1.0, x_d[k],
+                                   stream)
+
+    decode(head_step=head_step)          # eager runs of every token count
+    decode(head_step=head_step)          # graph captures
+    lm.lazymar_head_sync(hd, stream)
+    n_dec = max(1, min(args.steps, 2))
+    n0, f0 = lm.lazymar_head_counters(hd)
+    ms, _ = timed(lambda: decode(head_step=head_step), n_dec)
+    n1, f1 = lm.lazymar_head_counters(hd)
+    lm.lazymar_head_sync(hd, stream)
+    # the head alone, same calls
+    def heads_only():
+        for k in range(cfg["steps"]):
+            head_step(k)
+    ms_head, _ = timed(heads_only, n_dec)
+    hd.close()
+    return {"value": job_images_per_s(world, B, n_dec, ms), "unit": "images/s",
+            "ms_per_decode": ms / n_dec, "head_ms_per_decode": ms_head / n_dec,
+            "head_launches_per_decode": int((n1 - n0) // n_dec),
+            "head_tflops": (f1 - f0) / n_dec / (ms_head / n_dec / 1e3) / 1e12,
+            "head": {"width": hc["width"], "depth": hc["depth"], "n_steps": hc["n_steps"], "tokens_per_step": "B x n_new(k)",
+                     "note": "latents drawn by the head go to an output buffer; the next step's inputs stay the seeded ones"}}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -492,6 +566,7 @@ def main():
     ap.add_argument("--config", default="mar_b")
     ap.add_argument("--ratio", type=float, default=None, help="recompute ratio (default: the config's)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-head", action="store_true", help="skip the decode with the diffusion head")
     ap.add_argument("--select", default="least_similar", choices=sorted(SELECT_RULES),
                     help="token-selection strategy of the cached steps (Table 3; default: LazyMAR's)")
     ap.add_argument("--profile-case", choices=["gemm_layers", "attention_layers"], default=None,

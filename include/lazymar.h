@@ -250,9 +250,11 @@ lazymar_status lazymar_cfg_combine(int dtype, int mode, const void *z_cond, cons
  *   LAZYMAR_EPI_QKV      N = 3D: columns 0..D-1 -> out [M, D]; D..2D-1 ->
  *                        k_out[row_map[m], :]; 2D..3D-1 -> v_out[row_map[m], :]
  *                        (row_map NULL = identity; the cache scatter of Eq. 9)
+ *   LAZYMAR_EPI_SILU     out [M, ldo] dtype = SiLU(y) = y sigmoid(y)
  * flags: 0 automatic tile width, 1 force 128, 2 force 256, 3 force 192 (bf16;
  * a forced width that does not divide N falls back to 128). */
-enum { LAZYMAR_EPI_BIAS = 0, LAZYMAR_EPI_GELU = 1, LAZYMAR_EPI_RESIDUAL = 2, LAZYMAR_EPI_QKV = 3 };
+enum { LAZYMAR_EPI_BIAS = 0, LAZYMAR_EPI_GELU = 1, LAZYMAR_EPI_RESIDUAL = 2, LAZYMAR_EPI_QKV = 3,
+       LAZYMAR_EPI_SILU = 4 };
 lazymar_status lazymar_linear(int dtype, int epilogue, const void *a, const void *w,
                               const void *bias, int M, int N, int K, void *out, int ldo,
                               void *k_out, void *v_out, const int32_t *row_map, int flags,
@@ -302,6 +304,90 @@ lazymar_status lazymar_device_check(void *stream);
  * stream reports LAZYMAR_ERR_TIMEOUT (and clears it), and the device stays
  * usable. Returns INVALID_ARG outside the limit range. */
 lazymar_status lazymar_selftest_wait(int limit_us, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Diffusion head (Sec. 4.1: each decoded token's continuous latent is drawn
+ * by a per-token denoiser run for 100 diffusion steps of the standard sampler;
+ * its features z come from the transformer's final LayerNorm, a7).
+ *
+ * Denoiser (per token row r with latent x, training step t, feature z):
+ *   y = t_emb(t) + W_c z + b_c,  t_emb = Linear(SiLU(Linear(sinusoids(t))))
+ *   h = W_in x + b_in
+ *   per block: (shift, scale, gate) = W_ada SiLU(y) + b_ada
+ *              h += gate * MLP(LN(h) (1 + scale) + shift),  MLP = Linear, SiLU, Linear
+ *   (shift, scale) = W_fada SiLU(y) + b_fada
+ *   out = W_out (LN(h) (1 + scale) + shift) + b_out = [eps, v]  (2 token_dim)
+ * LN without gain or shift. Sampler: cosine schedule over n_train training
+ * steps, n_steps kept steps round(i (n_train - 1) / (n_steps - 1)); per kept
+ * step j = n_steps-1 .. 0 the network runs on (x, z_cond) and (x, z_uncond),
+ * eps = eps_u + gamma (eps_c - eps_u), v from the conditional run, and
+ *   x <- mean(x, eps) + [j > 0] exp(log_var(v) / 2) temperature noise
+ * with the Gaussian posterior mean and the learned-range log variance
+ * (frac = (v + 1) / 2 between log beta_j and the clipped log posterior
+ * variance). Weights are fp32 (host or device), stored as bf16 at create;
+ * the matrix products run on the tcgen05 tensor cores (width % 128 == 0,
+ * cond_dim % 64 == 0, freq_dim % 128 == 0).
+ * ------------------------------------------------------------------------ */
+typedef struct lazymar_head lazymar_head;
+typedef struct lazymar_head_config {
+  int token_dim;   /* latent width (16 for KL-16), 1..64 */
+  int cond_dim;    /* width of z (the transformer width) */
+  int z_dtype;     /* LAZYMAR_BF16 or LAZYMAR_F32: dtype of the z buffers */
+  int width;       /* denoiser width */
+  int depth;       /* residual blocks */
+  int freq_dim;    /* sinusoidal timestep features */
+  int n_train;     /* training steps of the noise schedule (1000) */
+  int n_steps;     /* sampling steps (100), 1..n_train */
+  int max_tokens;  /* tokens per lazymar_head_sample call */
+  float ln_eps;    /* LayerNorm epsilon (1e-6) */
+} lazymar_head_config;
+typedef struct lazymar_head_block_weights {
+  const float *ada_w, *ada_b;  /* [3 width, width], [3 width]: shift, scale, gate rows */
+  const float *w1, *b1;        /* [width, width], [width] */
+  const float *w2, *b2;        /* [width, width], [width] */
+} lazymar_head_block_weights;
+typedef struct lazymar_head_weights {
+  const float *t_w1, *t_b1;    /* [width, freq_dim], [width] */
+  const float *t_w2, *t_b2;    /* [width, width], [width] */
+  const float *c_w, *c_b;      /* [width, cond_dim], [width] */
+  const float *in_w, *in_b;    /* [width, token_dim], [width] */
+  const lazymar_head_block_weights *blocks;  /* depth entries */
+  const float *f_ada_w, *f_ada_b;  /* [2 width, width], [2 width]: shift, scale rows */
+  const float *out_w, *out_b;      /* [2 token_dim, width], [2 token_dim] */
+} lazymar_head_weights;
+
+/* Validates the configuration, copies the weights and precomputes the
+ * schedule and the time embeddings of the kept steps on the current device. */
+lazymar_status lazymar_head_create(const lazymar_head_config *cfg, const lazymar_head_weights *w,
+                                   lazymar_head **out);
+void lazymar_head_destroy(lazymar_head *hd);
+
+/* Draws the latents of the tokens decoded at one decoding step.
+ *   z      device [2B, n_img, cond_dim] (z_dtype): rows 0..B-1 the conditional
+ *          features of pairs 0..B-1, rows B..2B-1 the unconditional ones (the
+ *          z output of lazymar_full_step / lazymar_cached_step)
+ *   pos    [B, n_new] image positions decoded now (host or device), each in
+ *          0..n_img-1; token m = b n_new + k is pair b's position pos[b][k]
+ *   noise  [n_steps, B n_new, token_dim] fp32 (host or device): noise[0] the
+ *          starting latents, noise[i] the noise added after denoising step i
+ *   x_out  [B n_new, token_dim] fp32 (host or device)
+ * B n_new <= max_tokens. Asynchronous on `stream`; the sampling loop is
+ * captured into a CUDA graph per token count and replayed. Positions out of
+ * range raise LAZYMAR_ERR_DEVICE at the next check. */
+lazymar_status lazymar_head_sample(lazymar_head *hd, const void *z, int B, int n_img, const int32_t *pos,
+                                   int n_new, const float *noise, float gamma, float temperature,
+                                   float *x_out, void *stream);
+/* One guided network evaluation at kept step j (0 = last), for tests:
+ * out [2 B n_new, 2 token_dim] fp32 (host or device) = the network output of
+ * the conditional rows (0..M-1) and the unconditional rows (M..2M-1) for
+ * latents x [B n_new, token_dim] fp32. */
+lazymar_status lazymar_head_eval(lazymar_head *hd, const void *z, int B, int n_img, const int32_t *pos,
+                                 int n_new, const float *x, int j, float *out, void *stream);
+/* Kernel launches issued by this head so far (graph replays count their
+ * kernels), and the same for algorithmic flops. */
+lazymar_status lazymar_head_counters(lazymar_head *hd, long long *launches, double *flops);
+/* Waits for the head's work on `stream` and reports device errors. */
+lazymar_status lazymar_head_sync(lazymar_head *hd, void *stream);
 
 /* Per kernel class: launches, algorithmic flops and bytes, and (while
  * profiling is on) device time from CUDA events recorded around each launch on

@@ -22,7 +22,7 @@ INCLUDE = os.path.join(ROOT, "include")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O3",
                      "--expt-relaxed-constexpr", "-I", INCLUDE]
-SOURCES = ["lazymar_api.cu", "k_gemm.cu", "k_attention.cu", "k_rowwise.cu", "k_select.cu"]
+SOURCES = ["lazymar_api.cu", "k_gemm.cu", "k_attention.cu", "k_rowwise.cu", "k_select.cu", "k_head.cu"]
 
 
 def nvcc():

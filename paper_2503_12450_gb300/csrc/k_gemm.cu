@@ -39,10 +39,21 @@ __device__ __forceinline__ void epilogue_apply(const GemmEpi& e, int row, int co
       for (int i = 0; i < NC; ++i) v[i] = gelu_erf(v[i]);
       Vec<T, NC>::store(static_cast<T*>(e.out) + (size_t)row * e.ldo + col0, v);
       break;
+    case LAZYMAR_EPI_SILU:
+#pragma unroll
+      for (int i = 0; i < NC; ++i) v[i] = silu(v[i]);
+      Vec<T, NC>::store(static_cast<T*>(e.out) + (size_t)row * e.ldo + col0, v);
+      break;
     case LAZYMAR_EPI_RESIDUAL: {
       float* o = static_cast<float*>(e.out) + (size_t)row * e.ldo + col0;
       float r[NC];
       Vec<float, NC>::load(o, r);
+      if (e.gate) {
+        float g[NC];
+        Vec<T, NC>::load(static_cast<const T*>(e.gate) + (size_t)row * e.ldg + col0, g);
+#pragma unroll
+        for (int i = 0; i < NC; ++i) v[i] *= g[i];
+      }
 #pragma unroll
       for (int i = 0; i < NC; ++i) r[i] += v[i];
       Vec<float, NC>::store(o, r);
@@ -126,6 +137,15 @@ struct Cfg {
 __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
   return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
          ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// Gate of four consecutive residual columns (1 without a gate).
+__device__ __forceinline__ float4 gate4(const GemmEpi& e, int row, int col) {
+  if (!e.gate) return make_float4(1.f, 1.f, 1.f, 1.f);
+  const uint2 u = *reinterpret_cast<const uint2*>(static_cast<const bf16*>(e.gate) + (size_t)row * e.ldg + col);
+  const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+  const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+  return make_float4(a.x, a.y, b.x, b.y);
 }
 
 // Destination row pointer of a bf16 epilogue for tile row `row`, column `col`
@@ -358,11 +378,12 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
             const int row = rbase + lr;
             const float4 a = *reinterpret_cast<const float4*>(stg + lr * C::STG_PITCH + wq * 16);
             if (row < M) {
+              const float4 gg = tc::gate4(epi, row, col + wq * 4);
               float4 o;
-              o.x = cur[p].x + (a.x + bq.x);
-              o.y = cur[p].y + (a.y + bq.y);
-              o.z = cur[p].z + (a.z + bq.z);
-              o.w = cur[p].w + (a.w + bq.w);
+              o.x = fmaf(gg.x, a.x + bq.x, cur[p].x);
+              o.y = fmaf(gg.y, a.y + bq.y, cur[p].y);
+              o.z = fmaf(gg.z, a.z + bq.z, cur[p].z);
+              o.w = fmaf(gg.w, a.w + bq.w, cur[p].w);
               *reinterpret_cast<float4*>(res_base + (size_t)row * epi.ldo + col + wq * 4) = o;
             }
           }
@@ -396,11 +417,12 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
               const int row = rbase + lr;
               const float4 a = *reinterpret_cast<const float4*>(stg + lr * C::STG_PITCH + cq * 16);
               if (row < M) {
+                const float4 gg = tc::gate4(epi, row, col + h * 16 + cq * 4);
                 float4 o;
-                o.x = cur[h][p].x + (a.x + bq.x);
-                o.y = cur[h][p].y + (a.y + bq.y);
-                o.z = cur[h][p].z + (a.z + bq.z);
-                o.w = cur[h][p].w + (a.w + bq.w);
+                o.x = fmaf(gg.x, a.x + bq.x, cur[h][p].x);
+                o.y = fmaf(gg.y, a.y + bq.y, cur[h][p].y);
+                o.z = fmaf(gg.z, a.z + bq.z, cur[h][p].z);
+                o.w = fmaf(gg.w, a.w + bq.w, cur[h][p].w);
                 *reinterpret_cast<float4*>(res_base + (size_t)row * epi.ldo + col + h * 16 + cq * 4) = o;
               }
             }
@@ -417,6 +439,9 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
           if (epi.mode == LAZYMAR_EPI_GELU) {
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = gelu_erf(v[i]);
+          } else if (epi.mode == LAZYMAR_EPI_SILU) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = silu(v[i]);
           }
           uint4 pk[4];
           {
@@ -549,7 +574,11 @@ bool make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t o
 
 bool gemm_supported(int dtype, int M, int N, int K, const GemmEpi& epi, const char** why) {
   if (M < 0 || N <= 0 || K <= 0) { *why = "M >= 0, N > 0, K > 0 required"; return false; }
+  if (epi.mode < LAZYMAR_EPI_BIAS || epi.mode > LAZYMAR_EPI_SILU) { *why = "unknown epilogue"; return false; }
   if (epi.mode == LAZYMAR_EPI_QKV && (epi.D <= 0 || N != 3 * epi.D)) { *why = "QKV epilogue needs N = 3D"; return false; }
+  if (epi.gate && (epi.mode != LAZYMAR_EPI_RESIDUAL || epi.ldg < N || epi.ldg % 4 != 0)) {
+    *why = "a gate needs the residual epilogue and ldg >= N, ldg % 4 == 0"; return false;
+  }
   if (dtype == LAZYMAR_BF16) {
     if (K % 64 != 0) { *why = "bf16 GEMM needs K % 64 == 0"; return false; }
     if (N % 128 != 0) { *why = "bf16 GEMM needs N % 128 == 0"; return false; }

@@ -80,6 +80,12 @@ __device__ __forceinline__ float gelu_erf(float x) {
   return fmaf(-u, h, 0.5f * (x + fabsf(x)));
 }
 
+// SiLU(x) = x sigmoid(x) = x / (1 + 2^(-x log2 e)); for x below about -88
+// the denominator overflows to infinity and the quotient is -0.
+__device__ __forceinline__ float silu(float x) {
+  return __fdividef(x, 1.f + exp2_approx(-1.4426950408889634f * x));
+}
+
 // Three-input maximum (one instruction for two new values).
 __device__ __forceinline__ float fmax3(float a, float b, float c) {
   float d;
@@ -398,6 +404,10 @@ struct GemmEpi {
   void* v_out;          // QKV: V destination rows
   const int* row_map;   // QKV: destination row of K/V for row m (nullptr = m)
   int D;                // QKV: width of each of Q, K, V
+  // RESIDUAL only: out += gate * y with gate [M, ldg] in the GEMM dtype (the
+  // gated residual of an adaptive-LayerNorm block), or nullptr for out += y
+  const void* gate;
+  int ldg;
 };
 cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, int M, int N, int K,
                         const GemmEpi& epi, int flags);

@@ -16,7 +16,7 @@ LAZYMAR_F32, LAZYMAR_BF16 = 0, 1
 LAZYMAR_CRITERION_VALUE, LAZYMAR_CRITERION_FEATURE = 0, 1
 LAZYMAR_SELECT_LEAST_SIMILAR, LAZYMAR_SELECT_MOST_SIMILAR, LAZYMAR_SELECT_RANDOM = 0, 1, 2
 LAZYMAR_CFG_GUIDE, LAZYMAR_CFG_REFRESH, LAZYMAR_CFG_REUSE = 0, 1, 2
-LAZYMAR_EPI_BIAS, LAZYMAR_EPI_GELU, LAZYMAR_EPI_RESIDUAL, LAZYMAR_EPI_QKV = 0, 1, 2, 3
+LAZYMAR_EPI_BIAS, LAZYMAR_EPI_GELU, LAZYMAR_EPI_RESIDUAL, LAZYMAR_EPI_QKV, LAZYMAR_EPI_SILU = 0, 1, 2, 3, 4
 KERNEL_CLASSES = ["gemm", "attention", "layernorm", "select", "embed", "cfg", "other"]
 STATUS = {0: "LAZYMAR_OK", 1: "LAZYMAR_ERR_INVALID_ARG", 2: "LAZYMAR_ERR_OOM", 3: "LAZYMAR_ERR_CUDA",
           4: "LAZYMAR_ERR_STATE", 5: "LAZYMAR_ERR_TIMEOUT", 6: "LAZYMAR_ERR_UNSUPPORTED", 7: "LAZYMAR_ERR_DEVICE"}
@@ -61,6 +61,27 @@ class lazymar_stats(ctypes.Structure):
     _fields_ = [("k", lazymar_kernel_stats * 7)]
 
 
+class lazymar_head_config(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int) for n in ("token_dim", "cond_dim", "z_dtype", "width", "depth", "freq_dim",
+                                            "n_train", "n_steps", "max_tokens")] + [("ln_eps", ctypes.c_float)]
+
+
+HEAD_BLOCK_FIELDS = ("ada_w", "ada_b", "w1", "b1", "w2", "b2")
+
+
+class lazymar_head_block_weights(ctypes.Structure):
+    _fields_ = [(n, _FP) for n in HEAD_BLOCK_FIELDS]
+
+
+HEAD_FIELDS_A = ("t_w1", "t_b1", "t_w2", "t_b2", "c_w", "c_b", "in_w", "in_b")
+HEAD_FIELDS_B = ("f_ada_w", "f_ada_b", "out_w", "out_b")
+
+
+class lazymar_head_weights(ctypes.Structure):
+    _fields_ = [(n, _FP) for n in HEAD_FIELDS_A] + [("blocks", ctypes.POINTER(lazymar_head_block_weights))] + [
+        (n, _FP) for n in HEAD_FIELDS_B]
+
+
 _lib = None
 
 
@@ -96,6 +117,13 @@ def lib():
         "lazymar_reset_stats": (st, [vp]),
         "lazymar_status_string": (ctypes.c_char_p, [i]),
         "lazymar_last_error": (ctypes.c_char_p, []),
+        "lazymar_head_create": (st, [ctypes.POINTER(lazymar_head_config), ctypes.POINTER(lazymar_head_weights),
+                                     ctypes.POINTER(vp)]),
+        "lazymar_head_destroy": (None, [vp]),
+        "lazymar_head_sample": (st, [vp, vp, i, i, vp, i, vp, f, f, vp, vp]),
+        "lazymar_head_eval": (st, [vp, vp, i, i, vp, i, vp, i, vp, vp]),
+        "lazymar_head_counters": (st, [vp, ctypes.POINTER(ctypes.c_longlong), ctypes.POINTER(ctypes.c_double)]),
+        "lazymar_head_sync": (st, [vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -275,6 +303,76 @@ def lazymar_get_stats(h):
 
 def lazymar_reset_stats(h):
     _check(lib().lazymar_reset_stats(h.ptr))
+
+
+def lazymar_head_create(hc, cond_dim, token_dim, weights, max_tokens, z_dtype="bf16"):
+    """hc: dict with width, depth, freq_dim, n_train, n_steps (synth.head_config);
+    weights: dict as produced by synth.make_head_weights. Returns a HeadHandle."""
+    c = lazymar_head_config(int(token_dim), int(cond_dim),
+                            {"fp32": LAZYMAR_F32, "bf16": LAZYMAR_BF16}.get(z_dtype, z_dtype), int(hc["width"]),
+                            int(hc["depth"]), int(hc["freq_dim"]), int(hc["n_train"]), int(hc["n_steps"]),
+                            int(max_tokens), float(hc.get("ln_eps", 1e-6)))
+    keep = []
+
+    def p(a):
+        if hasattr(a, "data_ptr"):
+            keep.append(a)
+            return a.data_ptr()
+        import numpy as np
+        a = np.ascontiguousarray(a, dtype=np.float32)
+        keep.append(a)
+        return a.ctypes.data
+
+    w = lazymar_head_weights()
+    for n in HEAD_FIELDS_A + HEAD_FIELDS_B:
+        setattr(w, n, p(weights[n]))
+    blocks = (lazymar_head_block_weights * len(weights["blocks"]))()
+    for i, bw in enumerate(weights["blocks"]):
+        for n in HEAD_BLOCK_FIELDS:
+            setattr(blocks[i], n, p(bw[n]))
+    w.blocks = blocks
+    h = ctypes.c_void_p()
+    _check(lib().lazymar_head_create(ctypes.byref(c), ctypes.byref(w), ctypes.byref(h)))
+    return HeadHandle(h.value, c)
+
+
+def lazymar_head_sample(hd, z, B, n_img, pos, n_new, noise, gamma, temperature, x_out, stream=None):
+    _check(lib().lazymar_head_sample(hd.ptr, _ptr(z), int(B), int(n_img), _ptr(pos), int(n_new), _ptr(noise),
+                                     float(gamma), float(temperature), _ptr(x_out), _stream(stream)))
+
+
+def lazymar_head_eval(hd, z, B, n_img, pos, n_new, x, j, out, stream=None):
+    _check(lib().lazymar_head_eval(hd.ptr, _ptr(z), int(B), int(n_img), _ptr(pos), int(n_new), _ptr(x), int(j),
+                                   _ptr(out), _stream(stream)))
+
+
+def lazymar_head_counters(hd):
+    n, f = ctypes.c_longlong(), ctypes.c_double()
+    _check(lib().lazymar_head_counters(hd.ptr, ctypes.byref(n), ctypes.byref(f)))
+    return n.value, f.value
+
+
+def lazymar_head_sync(hd, stream=None):
+    _check(lib().lazymar_head_sync(hd.ptr, _stream(stream)))
+
+
+class HeadHandle:
+    """Owns a lazymar_head; destroyed with the object or by close()."""
+
+    def __init__(self, ptr, cfg):
+        self.ptr = ptr
+        self.cfg = cfg
+
+    def close(self):
+        if self.ptr:
+            lib().lazymar_head_destroy(self.ptr)
+            self.ptr = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
 
 
 def lazymar_status_string(status):

@@ -20,4 +20,8 @@ from .inputs import (  # noqa: F401
     tensor,
     similarity_inputs,
     distinct_rows,
+    HEAD_CONFIGS,
+    head_config,
+    make_head_weights,
+    make_head_noise,
 )

@@ -33,7 +33,8 @@ def test_exports_every_declared_symbol(lib):
     missing = [n for n in names if not hasattr(raw, n)]
     assert not missing, missing
     # and the binding exposes the same names
-    assert not [n for n in names if not hasattr(lm, n) and n not in ("lazymar_destroy", "lazymar_last_error")]
+    assert not [n for n in names if not hasattr(lm, n)
+                and n not in ("lazymar_destroy", "lazymar_last_error", "lazymar_head_destroy")]
 
 
 @pytest.mark.parametrize("k0,tau,tau_cfg,cond", [(4, 9, 9, True), (4, 9, 2, True), (3, 5, 5, True),
@@ -120,3 +121,33 @@ def test_component_argument_checks(lib):
     assert lib.lazymar_cfg_combine(1, 3, None, None, None, 1.0, 8, None, None, None) == 1
     assert lib.lazymar_attention(1, None, None, None, None, 1, 1, 1, 2, 96, None) == 6  # head width 96
     assert lib.lazymar_layernorm(1, None, None, None, None, None, 4, 200, 1e-6, None) == 6
+
+
+def _head_cfg(**kw):
+    c = dict(token_dim=16, cond_dim=768, z_dtype=lm.LAZYMAR_BF16, width=1024, depth=6, freq_dim=256, n_train=1000,
+             n_steps=100, max_tokens=64, ln_eps=1e-6)
+    c.update(kw)
+    return lm.lazymar_head_config(*[c[n] for n, _ in lm.lazymar_head_config._fields_])
+
+
+@pytest.mark.parametrize("bad,status", [
+    (dict(width=1000), 6), (dict(width=0), 6), (dict(cond_dim=100), 6), (dict(freq_dim=200), 6),
+    (dict(token_dim=0), 1), (dict(token_dim=65), 1), (dict(depth=0), 1), (dict(n_steps=0), 1),
+    (dict(n_steps=1001), 1), (dict(max_tokens=0), 1), (dict(z_dtype=7), 1), (dict(ln_eps=0.0), 1),
+])
+def test_head_create_rejects_bad_configs_before_touching_the_device(lib, bad, status):
+    w = lm.lazymar_head_weights()
+    w.blocks = (lm.lazymar_head_block_weights * 1)()
+    h = ctypes.c_void_p()
+    assert lib.lazymar_head_create(ctypes.byref(_head_cfg(**bad)), ctypes.byref(w), ctypes.byref(h)) == status
+    assert h.value is None
+
+
+def test_head_null_arguments_are_rejected(lib):
+    h = ctypes.c_void_p()
+    assert lib.lazymar_head_create(None, None, ctypes.byref(h)) == 1
+    assert lib.lazymar_head_sample(None, None, 1, 1, None, 1, None, 1.0, 1.0, None, None) == 1
+    assert lib.lazymar_head_eval(None, None, 1, 1, None, 1, None, 0, None, None) == 1
+    assert lib.lazymar_head_counters(None, None, None) == 1
+    assert lib.lazymar_head_sync(None, None) == 1
+    lib.lazymar_head_destroy(None)

@@ -4,6 +4,7 @@ import numpy as np
 import pytest
 
 import oracle as O
+from oracle import diffusion_head as HO
 import synth
 from paper_2503_12450_gb300 import lazymar as lm
 from _gpu import DT, TOL, dev, dev_int, empty, host, max_rel, sync, torch_cuda
@@ -178,11 +179,11 @@ def _linear_case(dtype, epi, M, N, K, flags, seed):
     ga, gw, gb = dev(a, dtype), dev(w, dtype), dev(b, dtype)
     ref = O.linear(a, w, b)
     out_dtype_tol = 1e-2 if dtype == "bf16" else 1e-4
-    if epi in (lm.LAZYMAR_EPI_BIAS, lm.LAZYMAR_EPI_GELU):
+    if epi in (lm.LAZYMAR_EPI_BIAS, lm.LAZYMAR_EPI_GELU, lm.LAZYMAR_EPI_SILU):
         out = empty((M, N), dtype)
         lm.lazymar_linear(DT[dtype], epi, ga, gw, gb, M, N, K, out, N, flags=flags)
         sync()
-        expect = ref if epi == lm.LAZYMAR_EPI_BIAS else O.gelu(ref)
+        expect = {lm.LAZYMAR_EPI_BIAS: ref, lm.LAZYMAR_EPI_GELU: O.gelu(ref), lm.LAZYMAR_EPI_SILU: HO.silu(ref)}[epi]
         assert max_rel(host(out), expect) < out_dtype_tol
     elif epi == lm.LAZYMAR_EPI_RESIDUAL:
         r0 = synth.tensor((M, N), seed + 3)
@@ -209,7 +210,7 @@ def _linear_case(dtype, epi, M, N, K, flags, seed):
 
 @pytest.mark.parametrize("M,N,K", GEMM_SHAPES)
 @pytest.mark.parametrize("epi", [lm.LAZYMAR_EPI_BIAS, lm.LAZYMAR_EPI_GELU, lm.LAZYMAR_EPI_RESIDUAL,
-                                 lm.LAZYMAR_EPI_QKV])
+                                 lm.LAZYMAR_EPI_QKV, lm.LAZYMAR_EPI_SILU])
 def test_linear_bf16_tcgen05(M, N, K, epi):
     if epi == lm.LAZYMAR_EPI_QKV and (N % 3 or (N // 3) % 32):
         pytest.skip("not a QKV shape")
@@ -219,7 +220,7 @@ def test_linear_bf16_tcgen05(M, N, K, epi):
 
 @pytest.mark.parametrize("M,N,K", [(1, 12, 8), (40, 768, 256), (160, 1024, 256), (77, 256, 1024)])
 @pytest.mark.parametrize("epi", [lm.LAZYMAR_EPI_BIAS, lm.LAZYMAR_EPI_GELU, lm.LAZYMAR_EPI_RESIDUAL,
-                                 lm.LAZYMAR_EPI_QKV])
+                                 lm.LAZYMAR_EPI_QKV, lm.LAZYMAR_EPI_SILU])
 def test_linear_fp32(M, N, K, epi):
     if epi == lm.LAZYMAR_EPI_QKV and (N % 3 or (N // 3) % 4):
         pytest.skip("not a QKV shape")
