@@ -459,7 +459,8 @@ def profile_case(args, cfg):
     """One launch of each kernel of a layer at the configuration's shapes, for a
     profiler: `gemm_layers` runs QKV, out-proj, fc1 and fc2 on all rows x T
     tokens and on the recomputed rows x N tokens; `attention_layers` runs the
-    recomputed-token and the full-layer attention."""
+    recomputed-token and the full-layer attention; `head` runs one eager
+    diffusion-head sampling call (100 steps) for 4 new tokens per pair."""
     import torch
     from paper_2503_12450_gb300 import lazymar as lm
     lm.lib()
@@ -485,6 +486,18 @@ def profile_case(args, cfg):
                     o = torch.empty(M, n, device=dev, dtype=torch.bfloat16)
                     lm.lazymar_linear(lm.LAZYMAR_BF16, epi, a, w, b, M, n, k, o, n)
                 torch.cuda.synchronize()
+    elif args.profile_case == "head":
+        B, n_img, td = cfg["batch"], cfg["n_img"], cfg["token_dim"]
+        hc = synth.head_config(HEAD_FOR[cfg["name"]])
+        n_new = 4
+        hd = lm.lazymar_head_create(hc, D, td, synth.make_head_weights(hc, D, td), max_tokens=B * n_new)
+        z = torch.randn(2 * B, n_img, D, device=dev).bfloat16()
+        pos = torch.stack([torch.randperm(n_img, device=dev)[:n_new] for _ in range(B)]).int()
+        noise = torch.randn(hc["n_steps"], B * n_new, td, device=dev)
+        x = torch.empty(B * n_new, td, device=dev)
+        lm.lazymar_head_sample(hd, z, B, n_img, pos, n_new, noise, GAMMA, 1.0, x)
+        lm.lazymar_head_sync(hd)
+        hd.close()
     else:
         for nq in (N, T):
             q = torch.randn(rows * nq, D, device=dev).bfloat16()
@@ -569,7 +582,7 @@ def main():
     ap.add_argument("--no-head", action="store_true", help="skip the decode with the diffusion head")
     ap.add_argument("--select", default="least_similar", choices=sorted(SELECT_RULES),
                     help="token-selection strategy of the cached steps (Table 3; default: LazyMAR's)")
-    ap.add_argument("--profile-case", choices=["gemm_layers", "attention_layers"], default=None,
+    ap.add_argument("--profile-case", choices=["gemm_layers", "attention_layers", "head"], default=None,
                     help="run each kernel of a layer once at the configuration's shapes (for ncu) and exit")
     args = ap.parse_args()
     cfg = synth.config(args.config)

@@ -90,7 +90,15 @@ constexpr int ATOM_K = 64;  // one 128-byte swizzle atom of bf16 along K (one TM
 // 32-column fp32 chunks (for short K, where the epilogue bounds the kernel, at
 // the cost of one pipeline stage); RESID_HALF stages 16-column halves and keeps
 // every stage (for long K, where the main loop bounds it).
-enum EpiKind { BF16OUT = 0, RESID_WIDE = 1, RESID_HALF = 2 };
+// RESID_WIDE_GATED is RESID_WIDE with a per-element gate on the product
+// (out += gate * y, the adaptive-LayerNorm residual of the diffusion head),
+// a separate instantiation so that the ungated kinds carry no gate code.
+// BF16OUT_SILU is BF16OUT with the SiLU activation, likewise separate.
+enum EpiKind { BF16OUT = 0, RESID_WIDE = 1, RESID_HALF = 2, RESID_WIDE_GATED = 3, BF16OUT_SILU = 4 };
+template <int EK>
+constexpr bool is_wide() { return EK == RESID_WIDE || EK == RESID_WIDE_GATED; }
+template <int EK>
+constexpr bool is_bf16out() { return EK == BF16OUT || EK == BF16OUT_SILU; }
 
 // BK: K per pipeline stage, one or two swizzle atoms. A 128-wide tile runs
 // 128-deep stages (two atoms, eight MMAs per barrier round trip): its
@@ -99,8 +107,8 @@ enum EpiKind { BF16OUT = 0, RESID_WIDE = 1, RESID_HALF = 2 };
 template <int BN, int EK, int BK>
 struct Cfg {
   static constexpr int ATOMS = BK / ATOM_K;
-  static constexpr int STAGES = BK == 128 ? (EK == RESID_WIDE ? 2 : 3)
-                                          : EK == RESID_WIDE ? (BN == 256 ? 3 : BN == 192 ? 4 : 5)
+  static constexpr int STAGES = BK == 128 ? (is_wide<EK>() ? 2 : 3)
+                                          : is_wide<EK>() ? (BN == 256 ? 3 : BN == 192 ? 4 : 5)
                                                              : (BN == 256 ? 4 : BN == 192 ? 5 : 6);
   static constexpr uint32_t A_BYTES = BM * BK * 2;
   static constexpr uint32_t B_BYTES = BN * BK * 2;
@@ -114,14 +122,14 @@ struct Cfg {
   // Epilogue warps: the bf16-output kinds use four (three for BN = 192) per
   // tensor-memory lane quarter, so more warps share a tile's conversion,
   // GELU and stores; the residual kinds, with more live registers, two.
-  static constexpr int EPI_WARPS = EK != BF16OUT ? 8 : (BN == 192 ? 12 : 16);
+  static constexpr int EPI_WARPS = !is_bf16out<EK>() ? 8 : (BN == 192 ? 12 : 16);
   static constexpr int THREADS = 64 + EPI_WARPS * 32;
   static constexpr int CHUNKS = BN / 32 / (EPI_WARPS / 4);  // 32-column chunks per warp and tile
   // Per-warp staging of 32 rows: bf16 rows of 64 bytes, 16-byte blocks
   // swizzled by row (conflict-free row-wise writes and column-block reads);
   // fp32 rows of 64 or 128 bytes padded by 16 bytes.
-  static constexpr uint32_t ROW_BYTES = EK == RESID_WIDE ? 128 : 64;
-  static constexpr uint32_t STG_PITCH = EK == BF16OUT ? 64 : ROW_BYTES + 16;
+  static constexpr uint32_t ROW_BYTES = is_wide<EK>() ? 128 : 64;
+  static constexpr uint32_t STG_PITCH = is_bf16out<EK>() ? 64 : ROW_BYTES + 16;
   static constexpr uint32_t STG_BYTES = 32 * STG_PITCH;
   static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + EPI_WARPS * STG_BYTES + 256;
   // Instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1),
@@ -139,9 +147,8 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
          ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
 
-// Gate of four consecutive residual columns (1 without a gate).
+// Gate of four consecutive residual columns.
 __device__ __forceinline__ float4 gate4(const GemmEpi& e, int row, int col) {
-  if (!e.gate) return make_float4(1.f, 1.f, 1.f, 1.f);
   const uint2 u = *reinterpret_cast<const uint2*>(static_cast<const bf16*>(e.gate) + (size_t)row * e.ldg + col);
   const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
   const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
@@ -167,7 +174,7 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
                         const __grid_constant__ CUtensorMap tmO2, int tma_out, int M, int N, int K, GemmEpi epi,
                         unsigned* err) {
   using C = tc::Cfg<BN, EK, BK>;
-  constexpr bool RESID = EK != tc::BF16OUT;
+  constexpr bool RESID = !tc::is_bf16out<EK>();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -342,7 +349,7 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
         }
       };
       if (EK == tc::RESID_HALF) load_res(n0 + c0 * 32);
-      if (EK == tc::RESID_WIDE) load_resw(n0 + c0 * 32);
+      if (tc::is_wide<EK>()) load_resw(n0 + c0 * 32);
       const bool ok = mbar_wait(&acc_full[buf], use, abort_flag, err);
       if (__any_sync(0xffffffffu, !ok)) break;
       tc_fence_after();
@@ -352,7 +359,7 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
         uint32_t r[32];
         tmem_ld32(tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN + c * 32), r);
         tmem_wait_ld();
-        if (EK == tc::RESID_WIDE) {
+        if (tc::is_wide<EK>()) {
           // whole 32-column fp32 chunk: 4 rows x 128 B per warp instruction
           float4* srow = reinterpret_cast<float4*>(stg + lane * C::STG_PITCH);
 #pragma unroll
@@ -378,12 +385,19 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
             const int row = rbase + lr;
             const float4 a = *reinterpret_cast<const float4*>(stg + lr * C::STG_PITCH + wq * 16);
             if (row < M) {
-              const float4 gg = tc::gate4(epi, row, col + wq * 4);
               float4 o;
-              o.x = fmaf(gg.x, a.x + bq.x, cur[p].x);
-              o.y = fmaf(gg.y, a.y + bq.y, cur[p].y);
-              o.z = fmaf(gg.z, a.z + bq.z, cur[p].z);
-              o.w = fmaf(gg.w, a.w + bq.w, cur[p].w);
+              if (EK == tc::RESID_WIDE_GATED) {
+                const float4 gg = tc::gate4(epi, row, col + wq * 4);
+                o.x = fmaf(gg.x, a.x + bq.x, cur[p].x);
+                o.y = fmaf(gg.y, a.y + bq.y, cur[p].y);
+                o.z = fmaf(gg.z, a.z + bq.z, cur[p].z);
+                o.w = fmaf(gg.w, a.w + bq.w, cur[p].w);
+              } else {
+                o.x = cur[p].x + (a.x + bq.x);
+                o.y = cur[p].y + (a.y + bq.y);
+                o.z = cur[p].z + (a.z + bq.z);
+                o.w = cur[p].w + (a.w + bq.w);
+              }
               *reinterpret_cast<float4*>(res_base + (size_t)row * epi.ldo + col + wq * 4) = o;
             }
           }
@@ -417,12 +431,11 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
               const int row = rbase + lr;
               const float4 a = *reinterpret_cast<const float4*>(stg + lr * C::STG_PITCH + cq * 16);
               if (row < M) {
-                const float4 gg = tc::gate4(epi, row, col + h * 16 + cq * 4);
                 float4 o;
-                o.x = fmaf(gg.x, a.x + bq.x, cur[h][p].x);
-                o.y = fmaf(gg.y, a.y + bq.y, cur[h][p].y);
-                o.z = fmaf(gg.z, a.z + bq.z, cur[h][p].z);
-                o.w = fmaf(gg.w, a.w + bq.w, cur[h][p].w);
+                o.x = cur[h][p].x + (a.x + bq.x);
+                o.y = cur[h][p].y + (a.y + bq.y);
+                o.z = cur[h][p].z + (a.z + bq.z);
+                o.w = cur[h][p].w + (a.w + bq.w);
                 *reinterpret_cast<float4*>(res_base + (size_t)row * epi.ldo + col + h * 16 + cq * 4) = o;
               }
             }
@@ -436,12 +449,12 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
           float v[32];
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]) + (epi.bias ? bv[i] : 0.f);
-          if (epi.mode == LAZYMAR_EPI_GELU) {
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = gelu_erf(v[i]);
-          } else if (epi.mode == LAZYMAR_EPI_SILU) {
+          if (EK == tc::BF16OUT_SILU) {
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = silu(v[i]);
+          } else if (epi.mode == LAZYMAR_EPI_GELU) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = gelu_erf(v[i]);
           }
           uint4 pk[4];
           {
@@ -617,7 +630,7 @@ static cudaError_t launch_tc(const Ctx& c, const void* A, const void* W, int M, 
   CUtensorMap to[3];
   std::memset(to, 0, sizeof to);
   int tma_out = 0;
-  if (EK == tc::BF16OUT && !(epi.mode == LAZYMAR_EPI_QKV && epi.row_map)) {
+  if (tc::is_bf16out<EK>() && !(epi.mode == LAZYMAR_EPI_QKV && epi.row_map)) {
     tma_out = 1;
     if (epi.mode == LAZYMAR_EPI_QKV) {
       const void* outs[3] = {epi.out, epi.k_out, epi.v_out};
@@ -669,24 +682,36 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
       }
     }
   }
-  const int ek = epi.mode != LAZYMAR_EPI_RESIDUAL ? tc::BF16OUT : (K < 2048 ? tc::RESID_WIDE : tc::RESID_HALF);
+  const int ek = epi.mode == LAZYMAR_EPI_SILU       ? tc::BF16OUT_SILU
+                 : epi.mode != LAZYMAR_EPI_RESIDUAL ? tc::BF16OUT
+                 : epi.gate                          ? tc::RESID_WIDE_GATED
+                 : K < 2048                          ? tc::RESID_WIDE
+                                                     : tc::RESID_HALF;
   if (bn == 192) {
     if (ek == tc::RESID_WIDE) return launch_tc<192, tc::RESID_WIDE, 64>(c, A, W, M, N, K, epi);
+    if (ek == tc::RESID_WIDE_GATED) return launch_tc<192, tc::RESID_WIDE_GATED, 64>(c, A, W, M, N, K, epi);
     if (ek == tc::RESID_HALF) return launch_tc<192, tc::RESID_HALF, 64>(c, A, W, M, N, K, epi);
+    if (ek == tc::BF16OUT_SILU) return launch_tc<192, tc::BF16OUT_SILU, 64>(c, A, W, M, N, K, epi);
     return launch_tc<192, tc::BF16OUT, 64>(c, A, W, M, N, K, epi);
   }
   if (bn == 256) {
     if (ek == tc::RESID_WIDE) return launch_tc<256, tc::RESID_WIDE, 64>(c, A, W, M, N, K, epi);
+    if (ek == tc::RESID_WIDE_GATED) return launch_tc<256, tc::RESID_WIDE_GATED, 64>(c, A, W, M, N, K, epi);
     if (ek == tc::RESID_HALF) return launch_tc<256, tc::RESID_HALF, 64>(c, A, W, M, N, K, epi);
+    if (ek == tc::BF16OUT_SILU) return launch_tc<256, tc::BF16OUT_SILU, 64>(c, A, W, M, N, K, epi);
     return launch_tc<256, tc::BF16OUT, 64>(c, A, W, M, N, K, epi);
   }
   if (K % 128 == 0) {
     if (ek == tc::RESID_WIDE) return launch_tc<128, tc::RESID_WIDE, 128>(c, A, W, M, N, K, epi);
+    if (ek == tc::RESID_WIDE_GATED) return launch_tc<128, tc::RESID_WIDE_GATED, 128>(c, A, W, M, N, K, epi);
     if (ek == tc::RESID_HALF) return launch_tc<128, tc::RESID_HALF, 128>(c, A, W, M, N, K, epi);
+    if (ek == tc::BF16OUT_SILU) return launch_tc<128, tc::BF16OUT_SILU, 128>(c, A, W, M, N, K, epi);
     return launch_tc<128, tc::BF16OUT, 128>(c, A, W, M, N, K, epi);
   }
   if (ek == tc::RESID_WIDE) return launch_tc<128, tc::RESID_WIDE, 64>(c, A, W, M, N, K, epi);
+  if (ek == tc::RESID_WIDE_GATED) return launch_tc<128, tc::RESID_WIDE_GATED, 64>(c, A, W, M, N, K, epi);
   if (ek == tc::RESID_HALF) return launch_tc<128, tc::RESID_HALF, 64>(c, A, W, M, N, K, epi);
+  if (ek == tc::BF16OUT_SILU) return launch_tc<128, tc::BF16OUT_SILU, 64>(c, A, W, M, N, K, epi);
   return launch_tc<128, tc::BF16OUT, 64>(c, A, W, M, N, K, epi);
 }
 
