@@ -147,9 +147,8 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
          ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
 
-// Gate of four consecutive residual columns.
-__device__ __forceinline__ float4 gate4(const GemmEpi& e, int row, int col) {
-  const uint2 u = *reinterpret_cast<const uint2*>(static_cast<const bf16*>(e.gate) + (size_t)row * e.ldg + col);
+// Four packed bf16 values as floats (the gates of four residual columns).
+__device__ __forceinline__ float4 bf16x4_to_f4(uint2 u) {
   const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
   const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
   return make_float4(a.x, a.y, b.x, b.y);
@@ -338,7 +337,9 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
           }
       };
       // RESID_WIDE layout: [pass] with 4 rows x 8 blocks of 16 bytes per pass
+      // (gated kind: the gates of the same elements, prefetched alike)
       float4 resw[8];
+      uint2 gatew[8];  // 4 bf16 gates each
       auto load_resw = [&](int col) {
         const int wr = lane >> 3, wq = lane & 7;
 #pragma unroll
@@ -346,6 +347,10 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
           const int row = rbase + p * 4 + wr;
           resw[p] = row < M ? *reinterpret_cast<const float4*>(res_base + (size_t)row * epi.ldo + col + wq * 4)
                             : make_float4(0.f, 0.f, 0.f, 0.f);
+          if (EK == tc::RESID_WIDE_GATED)
+            gatew[p] = row < M ? *reinterpret_cast<const uint2*>(static_cast<const bf16*>(epi.gate) +
+                                                                 (size_t)row * epi.ldg + col + wq * 4)
+                               : make_uint2(0u, 0u);
         }
       };
       if (EK == tc::RESID_HALF) load_res(n0 + c0 * 32);
@@ -376,8 +381,12 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
             bq = make_float4(bv[o], bv[o + 1], bv[o + 2], bv[o + 3]);
           }
           float4 cur[8];
+          uint2 curg[8];
 #pragma unroll
-          for (int p = 0; p < 8; ++p) cur[p] = resw[p];
+          for (int p = 0; p < 8; ++p) {
+            cur[p] = resw[p];
+            if (EK == tc::RESID_WIDE_GATED) curg[p] = gatew[p];
+          }
           if (c + 1 < c0 + CHUNKS) load_resw(col + 32);  // prefetch the next chunk
 #pragma unroll
           for (int p = 0; p < 8; ++p) {
@@ -387,7 +396,7 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
             if (row < M) {
               float4 o;
               if (EK == tc::RESID_WIDE_GATED) {
-                const float4 gg = tc::gate4(epi, row, col + wq * 4);
+                const float4 gg = tc::bf16x4_to_f4(curg[p]);
                 o.x = fmaf(gg.x, a.x + bq.x, cur[p].x);
                 o.y = fmaf(gg.y, a.y + bq.y, cur[p].y);
                 o.z = fmaf(gg.z, a.z + bq.z, cur[p].z);

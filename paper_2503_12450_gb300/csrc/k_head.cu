@@ -107,22 +107,30 @@ __global__ void __launch_bounds__(256) ln_mod_kernel(float* __restrict__ xh, con
   float4 v[VPL];
   float* xr = xh + (size_t)r * w;
   if (INPROJ) {
+    // latent index k outermost: each k issues VPL independent weight loads
     const float* xm = x + (size_t)(r < M ? r : r - M) * td;
 #pragma unroll
     for (int i = 0; i < VPL; ++i) {
-      const int c = 4 * (lane + 32 * i);
       float a[4];
-      load4_bf16(bin + c, a);
-      for (int k = 0; k < td; ++k) {
-        const float xk = xm[k];
-        float wk[4];
-        load4_bf16(win_t + (size_t)k * w + c, wk);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) a[q] = fmaf(xk, wk[q], a[q]);
-      }
+      load4_bf16(bin + 4 * (lane + 32 * i), a);
       v[i] = make_float4(a[0], a[1], a[2], a[3]);
-      reinterpret_cast<float4*>(xr)[lane + 32 * i] = v[i];
     }
+#pragma unroll 4
+    for (int k = 0; k < td; ++k) {
+      const float xk = xm[k];
+      const bf16* wrow = win_t + (size_t)k * w;
+#pragma unroll
+      for (int i = 0; i < VPL; ++i) {
+        float wk[4];
+        load4_bf16(wrow + 4 * (lane + 32 * i), wk);
+        v[i].x = fmaf(xk, wk[0], v[i].x);
+        v[i].y = fmaf(xk, wk[1], v[i].y);
+        v[i].z = fmaf(xk, wk[2], v[i].z);
+        v[i].w = fmaf(xk, wk[3], v[i].w);
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < VPL; ++i) reinterpret_cast<float4*>(xr)[lane + 32 * i] = v[i];
   } else {
 #pragma unroll
     for (int i = 0; i < VPL; ++i) v[i] = reinterpret_cast<const float4*>(xr)[lane + 32 * i];
@@ -217,13 +225,28 @@ __global__ void __launch_bounds__(FIN_THREADS) final_kernel(const float* __restr
       h[s * w + c] = fmaf((h[s * w + c] - mean) * rstd, 1.f + to_f(mr[scale_off + c]), to_f(mr[shift_off + c]));
     __syncthreads();
   }
-  // 2 rows x 2 td outputs, one warp per output at a time
+  // 2 rows x 2 td outputs, one warp per output at a time; each lane takes 8
+  // consecutive columns per 256 (one 16-byte weight load, w % 128 == 0)
   for (int k = warp; k < 4 * td; k += NW) {
     const int s = k / (2 * td), oc = k - s * 2 * td;
     const bf16* wr = wout + (size_t)oc * w;
-    float acc = 0.f;
-    for (int c = lane; c < w; c += 32) acc = fmaf(h[s * w + c], to_f(wr[c]), acc);
-    acc = warp_sum(acc);
+    const float* hs = h + s * w;
+    float acc0 = 0.f, acc1 = 0.f;
+    for (int c = 8 * lane; c < w; c += 256) {
+      float wv[8];
+      Vec<bf16, 8>::load(wr + c, wv);
+      const float4 h0 = *reinterpret_cast<const float4*>(hs + c);
+      const float4 h1 = *reinterpret_cast<const float4*>(hs + c + 4);
+      acc0 = fmaf(h0.x, wv[0], acc0);
+      acc1 = fmaf(h0.y, wv[1], acc1);
+      acc0 = fmaf(h0.z, wv[2], acc0);
+      acc1 = fmaf(h0.w, wv[3], acc1);
+      acc0 = fmaf(h1.x, wv[4], acc0);
+      acc1 = fmaf(h1.y, wv[5], acc1);
+      acc0 = fmaf(h1.z, wv[6], acc0);
+      acc1 = fmaf(h1.w, wv[7], acc1);
+    }
+    const float acc = warp_sum(acc0 + acc1);
     if (lane == 0) o[k] = acc + bout[oc];
   }
   __syncthreads();
