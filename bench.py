@@ -302,7 +302,7 @@ def run_ours(args, cfg):
     stream = torch.cuda.current_stream()
     dev_in = {"lat": lat, "mask": mask, "labels": labels, "guided": guided, "prio": prio, "keys": keys}
 
-    def decode(full_only=False, host=None, step_events=None, head_step=None):
+    def decode(full_only=False, host=None, step_events=None, head_step=None, after_step=None):
         for k in range(steps):
             full, reuse = plan[k]
             src = host if host is not None else dev_in
@@ -319,6 +319,8 @@ def run_ours(args, cfg):
                                        select_priority=p_k, select_keys=r_k)
             if head_step is not None:
                 head_step(k)
+            if after_step is not None:
+                after_step(k)
             if step_events is not None:
                 step_events[k][1].record(stream)
         if host is not None:
@@ -362,8 +364,20 @@ def run_ours(args, cfg):
     lm.lazymar_set_profiling(h, True)
     step_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
     kind_ms = {"full": [], "cached": [], "cached_reuse": []}
+    # GEMM flops and event time per step kind (statistics read after every step)
+    kind_gemm = {k: [0.0, 0.0] for k in kind_ms}
+    last = [lm.lazymar_get_stats(h)["gemm"]]
+
+    def after_step(k):
+        g = lm.lazymar_get_stats(h)["gemm"]
+        full, reuse = plan[k]
+        kind = "full" if full else ("cached_reuse" if reuse else "cached")
+        kind_gemm[kind][0] += g["flops"] - last[0]["flops"]
+        kind_gemm[kind][1] += g["ms"] - last[0]["ms"]
+        last[0] = g
+
     for _ in range(max(1, min(args.steps, 3))):
-        decode(step_events=step_ev)
+        decode(step_events=step_ev, after_step=after_step)
         torch.cuda.synchronize()
         for k in range(steps):
             full, reuse = plan[k]
@@ -420,6 +434,19 @@ def run_ours(args, cfg):
                          "share": round(v["ms"] / total_ms, 4) if total_ms else None,
                          "tflops": round(v["flops"] / (v["ms"] / 1e3) / 1e12, 2) if v["flops"] and v["ms"] else None,
                          "gbs": round(v["bytes"] / (v["ms"] / 1e3) / 1e9, 1) if v["ms"] else None}
+    peak_burst = pk["bf16_tflops"]
+
+    def gemm_rate(flops, ms):
+        if ms <= 0:
+            return None
+        tf = flops / (ms / 1e3) / 1e12
+        return {"tflops": round(tf, 1), "frac_of_sustained": round(tf / peak_tf, 4),
+                "frac_of_burst": round(tf / peak_burst, 4)}
+
+    gemm_by_kind = {k: gemm_rate(*v) for k, v in kind_gemm.items() if v[1] > 0}
+    cf = kind_gemm["cached"][0] + kind_gemm["cached_reuse"][0]
+    cm = kind_gemm["cached"][1] + kind_gemm["cached_reuse"][1]
+    gemm_by_kind["cached_steps_all"] = gemm_rate(cf, cm)
     traffic = None
     tpath = os.path.join(ROOT, "profiles", "gemm_traffic.json")  # captured on the MAR-B decode
     if cfg["name"] == "mar_b" and os.path.exists(tpath):
@@ -439,6 +466,7 @@ def run_ours(args, cfg):
                      "frac": (gemm_tflops / peak_tf) if gemm_tflops else None,
                      "peak_source": "%s bf16 sustained" % src, "traffic": traffic},
         "kernels": kernels,
+        "gemm_by_step_kind": gemm_by_kind,
         "e2e": {"value": e2e_images_per_s, "unit": "images/s", "h2d_bytes_per_step": int(h2d),
                 "d2h_bytes_per_step": int(d2h)},
         "gpu_launches": int(launches),
