@@ -13,8 +13,9 @@
 //                next LN + modulation                        (row-wise)
 //     final LN + modulation, output projection, guidance and the sampler
 //     update of x                                            (one CTA per token)
-// The loop is captured once per token count into a CUDA graph and replayed:
-// guidance scale and temperature are read from device memory, so they may
+// The loop runs eagerly on the first call with a given (z buffer, B, n_img,
+// n_new), is captured into a CUDA graph on the second and replayed after that.
+// The guidance scale and temperature are read from device memory, so they may
 // change between calls. The time embeddings of the kept steps depend on the
 // weights only and are computed once at create.
 #include <cmath>

@@ -139,3 +139,27 @@ def test_argument_checks():
         lm.lazymar_head_eval(h, dev(z, "bf16"), 1, 64, pos, 2, np.zeros((2, TD), np.float32), hc["n_steps"],
                              empty((4, 2 * TD)))
     h.close()
+
+
+@pytest.mark.parametrize("td,steps,B,n_new", [(4, 1, 2, 3), (64, 3, 1, 5), (16, 2, 3, 1)])
+def test_sampler_edge_shapes(td, steps, B, n_new):
+    """One kept step (no noise added at all), a few steps, latent widths 4 and 64."""
+    torch_cuda()
+    hc = S.head_config("tiny", n_steps=steps)
+    cond_dim, n_img = 128, 16
+    W = S.make_head_weights(hc, cond_dim, td, seed=61)
+    rng = np.random.default_rng(62)
+    z = S.round_bf16(rng.standard_normal((2 * B, n_img, cond_dim)).astype(np.float32))
+    pos = np.stack([rng.choice(n_img, n_new, replace=False) for _ in range(B)]).astype(np.int32)
+    h = lm.lazymar_head_create(hc, cond_dim, td, W, max_tokens=B * n_new)
+    M = B * n_new
+    noise = S.make_head_noise(steps, M, td, seed=63)
+    x = empty((M, td))
+    lm.lazymar_head_sample(h, dev(z, "bf16"), B, n_img, pos, n_new, noise, 2.0, 0.8, x)
+    lm.lazymar_head_sync(h)
+    zc, zu = z_rows(z, B, n_img, pos)
+    want = HO.sample(W, HO.Schedule(hc["n_train"], steps), zc, zu, noise, 2.0, 0.8)
+    got = host(x)
+    assert max_rel(got, want) < TOL["bf16"], max_rel(got, want)
+    assert min_cos(got, want) >= COS_MIN
+    h.close()
