@@ -117,7 +117,10 @@ class Schedule:
         pv = self.post_var.copy()
         if len(pv) > 1:
             pv[0] = pv[1]
-        self.post_log_var = np.log(pv)
+        # with a single kept step the posterior variance is 0 (log -inf); that
+        # step is the last one and adds no noise, so the value is never used
+        with np.errstate(divide="ignore"):
+            self.post_log_var = np.log(pv)
         self.coef_x0 = self.beta * np.sqrt(prev) / (1.0 - ab)
         self.coef_xt = (1.0 - prev) * np.sqrt(1.0 - self.beta) / (1.0 - ab)
 
