@@ -388,6 +388,14 @@ lazymar_status lazymar_head_eval(lazymar_head *hd, const void *z, int B, int n_i
 lazymar_status lazymar_head_counters(lazymar_head *hd, long long *launches, double *flops);
 /* Waits for the head's work on `stream` and reports device errors. */
 lazymar_status lazymar_head_sync(lazymar_head *hd, void *stream);
+/* The sampler's schedule as the head computes it (host only, no GPU): for
+ * kept steps j = 0..n_steps-1 (j = 0 the last denoising step),
+ * kept[j] = round(j (n_train - 1) / (n_steps - 1)) (ties to even), and
+ * consts[4 j + 0..3] = 1 / sqrt(1 - beta_j), beta_j / (sqrt(1 - beta_j)
+ * sqrt(1 - alpha_bar_j)), log beta_j and the clipped log posterior variance,
+ * so that mean = consts[0] x - consts[1] eps. Either output may be NULL.
+ * Returns INVALID_ARG unless 1 <= n_steps <= n_train. */
+lazymar_status lazymar_head_schedule(int n_train, int n_steps, int32_t *kept, float *consts);
 
 /* Per kernel class: launches, algorithmic flops and bytes, and (while
  * profiling is on) device time from CUDA events recorded around each launch on

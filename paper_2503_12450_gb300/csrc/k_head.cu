@@ -770,6 +770,24 @@ extern "C" lazymar_status lazymar_head_eval(lazymar_head* h, const void* z, int 
   return LAZYMAR_OK;
 }
 
+extern "C" lazymar_status lazymar_head_schedule(int n_train, int n_steps, int32_t* kept, float* consts) {
+  if (n_train < 1 || n_steps < 1 || n_steps > n_train)
+    return head_fail(LAZYMAR_ERR_INVALID_ARG, "need 1 <= n_steps <= n_train");
+  std::vector<int> k;
+  std::vector<hd::StepConst> sc;
+  make_schedule(n_train, n_steps, k, sc);
+  for (int j = 0; j < n_steps; ++j) {
+    if (kept) kept[j] = k[j];
+    if (consts) {
+      consts[4 * j] = sc[j].a_x;
+      consts[4 * j + 1] = sc[j].a_eps;
+      consts[4 * j + 2] = sc[j].log_beta;
+      consts[4 * j + 3] = sc[j].log_post;
+    }
+  }
+  return LAZYMAR_OK;
+}
+
 extern "C" lazymar_status lazymar_head_counters(lazymar_head* h, long long* launches, double* flops) {
   if (!h) return head_fail(LAZYMAR_ERR_INVALID_ARG, "NULL head");
   if (launches) *launches = h->launches;

@@ -124,6 +124,7 @@ def lib():
         "lazymar_head_eval": (st, [vp, vp, i, i, vp, i, vp, i, vp, vp]),
         "lazymar_head_counters": (st, [vp, ctypes.POINTER(ctypes.c_longlong), ctypes.POINTER(ctypes.c_double)]),
         "lazymar_head_sync": (st, [vp, vp]),
+        "lazymar_head_schedule": (st, [i, i, vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -350,6 +351,15 @@ def lazymar_head_counters(hd):
     n, f = ctypes.c_longlong(), ctypes.c_double()
     _check(lib().lazymar_head_counters(hd.ptr, ctypes.byref(n), ctypes.byref(f)))
     return n.value, f.value
+
+
+def lazymar_head_schedule(n_train, n_steps):
+    """(kept steps int32 [n_steps], constants float32 [n_steps, 4]) as the head computes them."""
+    import numpy as np
+    kept = np.zeros(n_steps, np.int32)
+    consts = np.zeros((n_steps, 4), np.float32)
+    _check(lib().lazymar_head_schedule(int(n_train), int(n_steps), kept.ctypes.data, consts.ctypes.data))
+    return kept, consts
 
 
 def lazymar_head_sync(hd, stream=None):

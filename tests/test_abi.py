@@ -151,3 +151,25 @@ def test_head_null_arguments_are_rejected(lib):
     assert lib.lazymar_head_counters(None, None, None) == 1
     assert lib.lazymar_head_sync(None, None) == 1
     lib.lazymar_head_destroy(None)
+
+
+@pytest.mark.parametrize("n_train,n_steps", [(1000, 100), (1000, 10), (1000, 1), (50, 50), (1001, 11), (4, 3), (6, 5)])
+def test_head_schedule_matches_the_oracle(lib, n_train, n_steps):
+    """The head's host-side schedule (kept steps, combined sampler constants)
+    against the oracle's schedule: steps exact, constants to fp32 rounding."""
+    import numpy as np
+    from oracle import diffusion_head as HO
+    kept, c = lm.lazymar_head_schedule(n_train, n_steps)
+    s = HO.Schedule(n_train, n_steps)
+    assert kept.tolist() == s.t.tolist()
+    a_x = s.coef_x0 / np.sqrt(s.alpha_bar) + s.coef_xt          # mean = a_x x - a_eps eps
+    a_eps = s.coef_x0 * np.sqrt(1.0 / s.alpha_bar - 1.0)
+    np.testing.assert_allclose(c[:, 0], a_x, rtol=2e-6)
+    np.testing.assert_allclose(c[:, 1], a_eps, rtol=2e-6)
+    np.testing.assert_allclose(c[:, 2], np.log(s.beta), rtol=2e-6)
+    np.testing.assert_allclose(c[:, 3], s.post_log_var, rtol=2e-6)
+
+
+def test_head_schedule_rejects_bad_sizes(lib):
+    assert lib.lazymar_head_schedule(10, 11, None, None) == 1
+    assert lib.lazymar_head_schedule(0, 0, None, None) == 1
