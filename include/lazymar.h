@@ -251,8 +251,9 @@ lazymar_status lazymar_cfg_combine(int dtype, int mode, const void *z_cond, cons
  *                        k_out[row_map[m], :]; 2D..3D-1 -> v_out[row_map[m], :]
  *                        (row_map NULL = identity; the cache scatter of Eq. 9)
  *   LAZYMAR_EPI_SILU     out [M, ldo] dtype = SiLU(y) = y sigmoid(y)
- * flags: 0 automatic tile width, 1 force 128, 2 force 256, 3 force 192 (bf16;
- * a forced width that does not divide N falls back to 128). */
+ * flags: 0 automatic tile width, 1 force 128, 2 force 256, 3 force 192, 4 force
+ * 64 (bf16; a forced width of 192 or 256 that does not divide N falls back to
+ * 128). */
 enum { LAZYMAR_EPI_BIAS = 0, LAZYMAR_EPI_GELU = 1, LAZYMAR_EPI_RESIDUAL = 2, LAZYMAR_EPI_QKV = 3,
        LAZYMAR_EPI_SILU = 4 };
 lazymar_status lazymar_linear(int dtype, int epilogue, const void *a, const void *w,

@@ -122,7 +122,7 @@ struct Cfg {
   // Epilogue warps: the bf16-output kinds use four (three for BN = 192) per
   // tensor-memory lane quarter, so more warps share a tile's conversion,
   // GELU and stores; the residual kinds, with more live registers, two.
-  static constexpr int EPI_WARPS = !is_bf16out<EK>() ? 8 : (BN == 192 ? 12 : 16);
+  static constexpr int EPI_WARPS = !is_bf16out<EK>() ? 8 : (BN == 192 ? 12 : BN == 64 ? 8 : 16);
   static constexpr int THREADS = 64 + EPI_WARPS * 32;
   static constexpr int CHUNKS = BN / 32 / (EPI_WARPS / 4);  // 32-column chunks per warp and tile
   // Per-warp staging of 32 rows: bf16 rows of 64 bytes, 16-byte blocks
@@ -671,17 +671,21 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
   // time of one tile. Relative tile times 187 : 243 : 256 for BN = 128 : 192 :
   // 256 (measured, one round of 128 x BN x 3072 tiles): a narrower tile does
   // proportionally less work per pipeline stage and runs well below the
-  // BN = 256 rate.
+  // BN = 256 rate. BN = 64 (153, on the line through the 128 and 256 points)
+  // wins only when the 128-wide tiles fit in one round with SMs to spare: the
+  // few-row GEMMs of the diffusion head.
   int bn = 128;
   if (flags == 2 && N % 256 == 0) {
     bn = 256;
   } else if (flags == 3 && N % 192 == 0) {
     bn = 192;
+  } else if (flags == 4) {
+    bn = 64;
   } else if (flags == 0) {
     const long mt = (M + tc::BM - 1) / tc::BM;
     long best = -1;
-    const int widths[3] = {256, 192, 128}, tile_time[3] = {256, 243, 187};
-    for (int i = 0; i < 3; ++i) {
+    const int widths[4] = {256, 192, 128, 64}, tile_time[4] = {256, 243, 187, 153};
+    for (int i = 0; i < 4; ++i) {
       if (N % widths[i] != 0) continue;
       const long rounds = (mt * (N / widths[i]) + c.num_sms - 1) / c.num_sms;
       const long cost = rounds * tile_time[i];
@@ -709,6 +713,20 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
     if (ek == tc::RESID_HALF) return launch_tc<256, tc::RESID_HALF, 64>(c, A, W, M, N, K, epi);
     if (ek == tc::BF16OUT_SILU) return launch_tc<256, tc::BF16OUT_SILU, 64>(c, A, W, M, N, K, epi);
     return launch_tc<256, tc::BF16OUT, 64>(c, A, W, M, N, K, epi);
+  }
+  if (bn == 64) {
+    if (K % 128 == 0) {
+      if (ek == tc::RESID_WIDE) return launch_tc<64, tc::RESID_WIDE, 128>(c, A, W, M, N, K, epi);
+      if (ek == tc::RESID_WIDE_GATED) return launch_tc<64, tc::RESID_WIDE_GATED, 128>(c, A, W, M, N, K, epi);
+      if (ek == tc::RESID_HALF) return launch_tc<64, tc::RESID_HALF, 128>(c, A, W, M, N, K, epi);
+      if (ek == tc::BF16OUT_SILU) return launch_tc<64, tc::BF16OUT_SILU, 128>(c, A, W, M, N, K, epi);
+      return launch_tc<64, tc::BF16OUT, 128>(c, A, W, M, N, K, epi);
+    }
+    if (ek == tc::RESID_WIDE) return launch_tc<64, tc::RESID_WIDE, 64>(c, A, W, M, N, K, epi);
+    if (ek == tc::RESID_WIDE_GATED) return launch_tc<64, tc::RESID_WIDE_GATED, 64>(c, A, W, M, N, K, epi);
+    if (ek == tc::RESID_HALF) return launch_tc<64, tc::RESID_HALF, 64>(c, A, W, M, N, K, epi);
+    if (ek == tc::BF16OUT_SILU) return launch_tc<64, tc::BF16OUT_SILU, 64>(c, A, W, M, N, K, epi);
+    return launch_tc<64, tc::BF16OUT, 64>(c, A, W, M, N, K, epi);
   }
   if (K % 128 == 0) {
     if (ek == tc::RESID_WIDE) return launch_tc<128, tc::RESID_WIDE, 128>(c, A, W, M, N, K, epi);

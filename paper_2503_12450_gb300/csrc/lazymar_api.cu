@@ -743,7 +743,7 @@ extern "C" lazymar_status lazymar_linear(int dtype, int epilogue, const void* a,
                                          int N, int K, void* out, int ldo, void* k_out, void* v_out,
                                          const int32_t* row_map, int flags, void* stream) {
   if (epilogue < LAZYMAR_EPI_BIAS || epilogue > LAZYMAR_EPI_SILU) return fail(LAZYMAR_ERR_INVALID_ARG, "epilogue");
-  if (flags < 0 || flags > 3) return fail(LAZYMAR_ERR_INVALID_ARG, "flags");
+  if (flags < 0 || flags > 4) return fail(LAZYMAR_ERR_INVALID_ARG, "flags");
   GemmEpi e{epilogue, bias, out, ldo, k_out, v_out, row_map, epilogue == LAZYMAR_EPI_QKV ? N / 3 : 0};
   const char* why = "";
   if (!gemm_supported(dtype, M, N, K, e, &why)) return fail(LAZYMAR_ERR_UNSUPPORTED, why);

@@ -214,7 +214,7 @@ def _linear_case(dtype, epi, M, N, K, flags, seed):
 def test_linear_bf16_tcgen05(M, N, K, epi):
     if epi == lm.LAZYMAR_EPI_QKV and (N % 3 or (N // 3) % 32):
         pytest.skip("not a QKV shape")
-    for flags in [1] + ([2] if N % 256 == 0 else []) + ([3] if N % 192 == 0 else []):
+    for flags in [1, 4] + ([2] if N % 256 == 0 else []) + ([3] if N % 192 == 0 else []):
         _linear_case("bf16", epi, M, N, K, flags, seed=M + N + K + epi)
 
 
