@@ -72,18 +72,22 @@ __global__ void __launch_bounds__(256) gather_z_kernel(const TZ* __restrict__ z,
   for (int c = lane; c < D; c += 32) out[(size_t)r * D + c] = __float2bfloat16_rn(to_f(z[src + c]));
 }
 
-// sy[r] = SiLU(t_emb_j + c_emb[r]), 8 bf16 per thread.
-__global__ void __launch_bounds__(256) cond_silu_kernel(const bf16* __restrict__ temb, const bf16* __restrict__ cemb,
-                                                        bf16* __restrict__ sy, int R, int w) {
+// For cnt kept steps j0, j0 - 1, ..: sy[k R + r] = SiLU(t_emb[j0 - k] +
+// c_emb[r]), 8 bf16 per thread.
+__global__ void __launch_bounds__(256) cond_silu_kernel(const bf16* __restrict__ temb, int j0, int cnt,
+                                                        const bf16* __restrict__ cemb, bf16* __restrict__ sy, int R,
+                                                        int w) {
   pdl_wait();
   pdl_trigger();
   const int w8 = w / 8;
-  const int n = R * w8;
+  const int per = R * w8;
+  const int n = cnt * per;
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
-    const int c8 = i % w8;
+    const int k = i / per, rem = i - k * per;
+    const int c8 = rem % w8;
     float a[8], b[8];
-    Vec<bf16, 8>::load(temb + c8 * 8, a);
-    Vec<bf16, 8>::load(cemb + (size_t)i * 8, b);
+    Vec<bf16, 8>::load(temb + (size_t)(j0 - k) * w + c8 * 8, a);
+    Vec<bf16, 8>::load(cemb + (size_t)rem * 8, b);
 #pragma unroll
     for (int k = 0; k < 8; ++k) a[k] = silu(a[k] + b[k]);
     Vec<bf16, 8>::store(sy + (size_t)i * 8, a);
@@ -317,6 +321,7 @@ bool width_ok(int w) {
 struct lazymar_head {
   lazymar_head_config cfg{};
   int dev = 0, num_sms = 0, w = 0, td = 0, nmod = 0;
+  int chunk = 1;  // kept steps whose modulations are computed by one GEMM
   uint8_t* arena = nullptr;
   // weights (bf16 unless noted)
   bf16 *t_w1 = nullptr, *t_b1 = nullptr, *t_w2 = nullptr, *t_b2 = nullptr, *c_w = nullptr, *c_b = nullptr;
@@ -364,35 +369,37 @@ lazymar_status hgemm(lazymar_head* h, const Ctx& c, const void* A, const void* W
 }
 
 template <int VPL>
-cudaError_t launch_ln_mod_t(const Ctx& c, lazymar_head* h, bool inproj, int R, int M, int shift_off, int scale_off) {
+cudaError_t launch_ln_mod_t(const Ctx& c, lazymar_head* h, const bf16* mod, bool inproj, int R, int M, int shift_off,
+                            int scale_off) {
   const unsigned grid = (unsigned)((R + 7) / 8);
   if (inproj)
     return launch_pdl(hd::ln_mod_kernel<VPL, true>, dim3(grid), dim3(256), 0, c.stream, h->xh, (const float*)h->x,
-                      (const bf16*)h->in_wt, (const bf16*)h->in_b, (const bf16*)h->mod, h->nmod, shift_off, scale_off,
-                      h->hb, R, M, h->td, h->cfg.ln_eps);
+                      (const bf16*)h->in_wt, (const bf16*)h->in_b, mod, h->nmod, shift_off, scale_off, h->hb, R, M,
+                      h->td, h->cfg.ln_eps);
   return launch_pdl(hd::ln_mod_kernel<VPL, false>, dim3(grid), dim3(256), 0, c.stream, h->xh, (const float*)h->x,
-                    (const bf16*)h->in_wt, (const bf16*)h->in_b, (const bf16*)h->mod, h->nmod, shift_off, scale_off,
-                    h->hb, R, M, h->td, h->cfg.ln_eps);
+                    (const bf16*)h->in_wt, (const bf16*)h->in_b, mod, h->nmod, shift_off, scale_off, h->hb, R, M,
+                    h->td, h->cfg.ln_eps);
 }
 
-cudaError_t launch_ln_mod(const Ctx& c, lazymar_head* h, bool inproj, int R, int M, int shift_off, int scale_off) {
+cudaError_t launch_ln_mod(const Ctx& c, lazymar_head* h, const bf16* mod, bool inproj, int R, int M, int shift_off,
+                          int scale_off) {
   switch (h->w / 128) {
-    case 1: return launch_ln_mod_t<1>(c, h, inproj, R, M, shift_off, scale_off);
-    case 2: return launch_ln_mod_t<2>(c, h, inproj, R, M, shift_off, scale_off);
-    case 3: return launch_ln_mod_t<3>(c, h, inproj, R, M, shift_off, scale_off);
-    case 4: return launch_ln_mod_t<4>(c, h, inproj, R, M, shift_off, scale_off);
-    case 5: return launch_ln_mod_t<5>(c, h, inproj, R, M, shift_off, scale_off);
-    case 6: return launch_ln_mod_t<6>(c, h, inproj, R, M, shift_off, scale_off);
-    case 7: return launch_ln_mod_t<7>(c, h, inproj, R, M, shift_off, scale_off);
-    case 8: return launch_ln_mod_t<8>(c, h, inproj, R, M, shift_off, scale_off);
-    case 9: return launch_ln_mod_t<9>(c, h, inproj, R, M, shift_off, scale_off);
-    case 10: return launch_ln_mod_t<10>(c, h, inproj, R, M, shift_off, scale_off);
-    case 11: return launch_ln_mod_t<11>(c, h, inproj, R, M, shift_off, scale_off);
-    case 12: return launch_ln_mod_t<12>(c, h, inproj, R, M, shift_off, scale_off);
-    case 13: return launch_ln_mod_t<13>(c, h, inproj, R, M, shift_off, scale_off);
-    case 14: return launch_ln_mod_t<14>(c, h, inproj, R, M, shift_off, scale_off);
-    case 15: return launch_ln_mod_t<15>(c, h, inproj, R, M, shift_off, scale_off);
-    case 16: return launch_ln_mod_t<16>(c, h, inproj, R, M, shift_off, scale_off);
+    case 1: return launch_ln_mod_t<1>(c, h, mod, inproj, R, M, shift_off, scale_off);
+    case 2: return launch_ln_mod_t<2>(c, h, mod, inproj, R, M, shift_off, scale_off);
+    case 3: return launch_ln_mod_t<3>(c, h, mod, inproj, R, M, shift_off, scale_off);
+    case 4: return launch_ln_mod_t<4>(c, h, mod, inproj, R, M, shift_off, scale_off);
+    case 5: return launch_ln_mod_t<5>(c, h, mod, inproj, R, M, shift_off, scale_off);
+    case 6: return launch_ln_mod_t<6>(c, h, mod, inproj, R, M, shift_off, scale_off);
+    case 7: return launch_ln_mod_t<7>(c, h, mod, inproj, R, M, shift_off, scale_off);
+    case 8: return launch_ln_mod_t<8>(c, h, mod, inproj, R, M, shift_off, scale_off);
+    case 9: return launch_ln_mod_t<9>(c, h, mod, inproj, R, M, shift_off, scale_off);
+    case 10: return launch_ln_mod_t<10>(c, h, mod, inproj, R, M, shift_off, scale_off);
+    case 11: return launch_ln_mod_t<11>(c, h, mod, inproj, R, M, shift_off, scale_off);
+    case 12: return launch_ln_mod_t<12>(c, h, mod, inproj, R, M, shift_off, scale_off);
+    case 13: return launch_ln_mod_t<13>(c, h, mod, inproj, R, M, shift_off, scale_off);
+    case 14: return launch_ln_mod_t<14>(c, h, mod, inproj, R, M, shift_off, scale_off);
+    case 15: return launch_ln_mod_t<15>(c, h, mod, inproj, R, M, shift_off, scale_off);
+    case 16: return launch_ln_mod_t<16>(c, h, mod, inproj, R, M, shift_off, scale_off);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -412,28 +419,36 @@ lazymar_status prologue(lazymar_head* h, const Ctx& c, const void* z, int B, int
                GemmEpi{LAZYMAR_EPI_BIAS, h->c_b, h->cemb, h->w, nullptr, nullptr, nullptr, 0});
 }
 
-// One network evaluation at kept step j on rows [x; x] with conditions
-// c_emb; ends with the final kernel (sampler update, or raw outputs to
-// eval_out).
-lazymar_status network(lazymar_head* h, const Ctx& c, int M, int j, bool done, float* eval_out) {
-  const int R = 2 * M, w = h->w, depth = h->cfg.depth, td = h->td;
+// The modulations (all blocks' shift, scale, gate and the final shift,
+// scale) of cnt kept steps j0, j0 - 1, .. for the R rows, in one GEMM:
+// step j0 - k's rows start at h->mod + k R nmod. They depend on t_emb and
+// c_emb only, not on x.
+lazymar_status modulations(lazymar_head* h, const Ctx& c, int M, int j0, int cnt) {
+  const int R = 2 * M, w = h->w;
   HD_TRY(hlaunch(h, 0.0, "head condition", [&] {
-    const int n = R * (w / 8);
-    int blocks = (n + 255) / 256;
-    if (blocks > 4 * h->num_sms) blocks = 4 * h->num_sms;
-    return launch_pdl(hd::cond_silu_kernel, dim3(blocks), dim3(256), 0, c.stream,
-                      (const bf16*)(h->temb + (size_t)j * w), (const bf16*)h->cemb, h->sy, R, w);
+    const long long n = (long long)cnt * R * (w / 8);
+    long long blocks = (n + 255) / 256;
+    if (blocks > 8LL * h->num_sms) blocks = 8LL * h->num_sms;
+    return launch_pdl(hd::cond_silu_kernel, dim3((unsigned)blocks), dim3(256), 0, c.stream, (const bf16*)h->temb, j0,
+                      cnt, (const bf16*)h->cemb, h->sy, R, w);
   }));
-  HD_TRY(hgemm(h, c, h->sy, h->ada_w, R, h->nmod, w,
-               GemmEpi{LAZYMAR_EPI_BIAS, h->ada_b, h->mod, h->nmod, nullptr, nullptr, nullptr, 0}));
+  return hgemm(h, c, h->sy, h->ada_w, cnt * R, h->nmod, w,
+               GemmEpi{LAZYMAR_EPI_BIAS, h->ada_b, h->mod, h->nmod, nullptr, nullptr, nullptr, 0});
+}
+
+// One network evaluation at kept step j on rows [x; x] with its modulations
+// `mod` (R rows of nmod); ends with the final kernel (sampler update, or raw
+// outputs to eval_out).
+lazymar_status network(lazymar_head* h, const Ctx& c, int M, int j, const bf16* mod, bool done, float* eval_out) {
+  const int R = 2 * M, w = h->w, depth = h->cfg.depth, td = h->td;
   for (int b = 0; b < depth; ++b) {
     HD_TRY(hlaunch(h, b == 0 ? 2.0 * R * td * w : 0.0, "head layernorm", [&] {
-      return launch_ln_mod(c, h, b == 0, R, M, 3 * w * b, 3 * w * b + w);
+      return launch_ln_mod(c, h, mod, b == 0, R, M, 3 * w * b, 3 * w * b + w);
     }));
     HD_TRY(hgemm(h, c, h->hb, h->w1[b], R, w, w,
                  GemmEpi{LAZYMAR_EPI_SILU, h->b1[b], h->u, w, nullptr, nullptr, nullptr, 0}));
     GemmEpi e2{LAZYMAR_EPI_RESIDUAL, h->b2[b], h->xh, w, nullptr, nullptr, nullptr, 0};
-    e2.gate = h->mod + 3 * w * b + 2 * w;
+    e2.gate = mod + 3 * w * b + 2 * w;
     e2.ldg = h->nmod;
     HD_TRY(hgemm(h, c, h->u, h->w2[b], R, w, w, e2));
   }
@@ -441,9 +456,9 @@ lazymar_status network(lazymar_head* h, const Ctx& c, int M, int j, bool done, f
   const int fshift = 3 * w * depth, fscale = fshift + w;
   const size_t smem = (size_t)(2 * w + 4 * td + 2 * (hd::FIN_THREADS / 32)) * sizeof(float);
   return hlaunch(h, 2.0 * R * 2 * td * w, "head final", [&] {
-    return launch_pdl(hd::final_kernel, dim3(M), dim3(hd::FIN_THREADS), smem, c.stream, (const float*)h->xh,
-                      (const bf16*)h->mod, h->nmod, fshift, fscale, (const bf16*)h->out_w, (const float*)h->out_b, M,
-                      w, td, h->cfg.ln_eps, sc, (const float*)h->params, h->x,
+    return launch_pdl(hd::final_kernel, dim3(M), dim3(hd::FIN_THREADS), smem, c.stream, (const float*)h->xh, mod,
+                      h->nmod, fshift, fscale, (const bf16*)h->out_w, (const float*)h->out_b, M, w, td,
+                      h->cfg.ln_eps, sc, (const float*)h->params, h->x,
                       (const float*)(h->noise + (size_t)(h->cfg.n_steps - 1 - j + (sc.last ? 0 : 1)) * M * td),
                       done ? h->x_done : nullptr, eval_out);
   });
@@ -454,7 +469,12 @@ lazymar_status sample_body(lazymar_head* h, const Ctx& c, const void* z, int B, 
   const int M = B * n_new, td = h->td;
   HD_TRY(prologue(h, c, z, B, n_img, n_new, M));
   HD_CUDA(cudaMemcpyAsync(h->x, h->noise, (size_t)M * td * sizeof(float), cudaMemcpyDeviceToDevice, c.stream));
-  for (int j = h->cfg.n_steps - 1; j >= 0; --j) HD_TRY(network(h, c, M, j, j == 0, nullptr));
+  for (int j0 = h->cfg.n_steps - 1; j0 >= 0; j0 -= h->chunk) {
+    const int cnt = j0 + 1 < h->chunk ? j0 + 1 : h->chunk;
+    HD_TRY(modulations(h, c, M, j0, cnt));
+    for (int k = 0; k < cnt; ++k)
+      HD_TRY(network(h, c, M, j0 - k, h->mod + (size_t)k * 2 * M * h->nmod, j0 - k == 0, nullptr));
+  }
   return LAZYMAR_OK;
 }
 
@@ -586,6 +606,17 @@ extern "C" lazymar_status lazymar_head_create(const lazymar_head_config* cfg, co
 
   const size_t W = c.width, F = c.freq_dim, CD = c.cond_dim, TD = c.token_dim, NM = h->nmod, NS = c.n_steps;
   const size_t R = 2 * (size_t)c.max_tokens, MT = c.max_tokens;
+  // modulations of up to `chunk` kept steps at once, within 1 GB and with
+  // fewer than 2^31 rows x columns per GEMM
+  {
+    const double per_step = (double)R * NM;
+    long long ch = (long long)(1e9 / (2.0 * per_step));
+    const long long cap = (long long)((double)(1ll << 31) / per_step);
+    if (ch > cap) ch = cap;
+    if (ch > c.n_steps) ch = c.n_steps;
+    h->chunk = ch < 1 ? 1 : (int)ch;
+  }
+  const size_t CH = (size_t)h->chunk;
   size_t off = 0;
   auto take = [&](size_t bytes) {
     const size_t o = off;
@@ -602,7 +633,7 @@ extern "C" lazymar_status lazymar_head_create(const lazymar_head_config* cfg, co
   const size_t o_temb = take(NS * W * 2), o_sin = take(NS * F * 2), o_t1 = take(NS * W * 2), o_kept = take(NS * 4);
   const size_t o_pos = take(MT * 4), o_noise = take(NS * MT * TD * 4), o_x = take(MT * TD * 4), o_xd = take(MT * TD * 4),
                o_xh = take(R * W * 4), o_eval = take(R * 2 * TD * 4), o_par = take(2 * 4), o_zg = take(R * CD * 2),
-               o_cemb = take(R * W * 2), o_sy = take(R * W * 2), o_mod = take(R * NM * 2), o_hb = take(R * W * 2),
+               o_cemb = take(R * W * 2), o_sy = take(CH * R * W * 2), o_mod = take(CH * R * NM * 2), o_hb = take(R * W * 2),
                o_u = take(R * W * 2), o_err = take(4);
   e = cudaMalloc(&h->arena, off);
   if (e != cudaSuccess) {
@@ -765,7 +796,8 @@ extern "C" lazymar_status lazymar_head_eval(lazymar_head* h, const void* z, int 
   HD_CUDA(cudaMemcpyAsync(h->x, x, (size_t)M * h->td * 4, cudaMemcpyDefault, st));
   const Ctx c{st, h->err, h->num_sms};
   HD_TRY(prologue(h, c, z, B, n_img, n_new, M));
-  HD_TRY(network(h, c, M, j, false, h->eval));
+  HD_TRY(modulations(h, c, M, j, 1));
+  HD_TRY(network(h, c, M, j, h->mod, false, h->eval));
   HD_CUDA(cudaMemcpyAsync(out, h->eval, (size_t)2 * M * 2 * h->td * 4, cudaMemcpyDefault, st));
   return LAZYMAR_OK;
 }
