@@ -30,12 +30,15 @@
 namespace lm {
 namespace hd {
 
-// Four consecutive bf16 values (8-byte aligned) as floats.
-__device__ __forceinline__ void load4_bf16(const bf16* p, float* v) {
-  const uint2 u = *reinterpret_cast<const uint2*>(p);
+// Four packed bf16 values as floats.
+__device__ __forceinline__ void unpack4_bf16(uint2 u, float* v) {
   const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
   const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
   v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y;
+}
+// Four consecutive bf16 values (8-byte aligned) as floats.
+__device__ __forceinline__ void load4_bf16(const bf16* p, float* v) {
+  unpack4_bf16(*reinterpret_cast<const uint2*>(p), v);
 }
 
 // Sinusoidal features of the kept training steps: [cos(t f_i), sin(t f_i)],
@@ -111,6 +114,15 @@ __global__ void __launch_bounds__(256) ln_mod_kernel(float* __restrict__ xh, con
   constexpr int w = 128 * VPL;
   float4 v[VPL];
   float* xr = xh + (size_t)r * w;
+  // the modulation does not depend on the row: its loads go out first
+  const bf16* mr = mod + (size_t)r * ldm;
+  uint2 shp[VPL], scp[VPL];
+#pragma unroll
+  for (int i = 0; i < VPL; ++i) {
+    const int c = 4 * (lane + 32 * i);
+    shp[i] = *reinterpret_cast<const uint2*>(mr + shift_off + c);
+    scp[i] = *reinterpret_cast<const uint2*>(mr + scale_off + c);
+  }
   if (INPROJ) {
     // latent index k outermost: each k issues VPL independent weight loads
     const float* xm = x + (size_t)(r < M ? r : r - M) * td;
@@ -151,13 +163,12 @@ __global__ void __launch_bounds__(256) ln_mod_kernel(float* __restrict__ xh, con
     q += (a * a + b * b) + (c * c + d * d);
   }
   const float rstd = rsqrtf(warp_sum(q) * (1.f / w) + eps);
-  const bf16* mr = mod + (size_t)r * ldm;
 #pragma unroll
   for (int i = 0; i < VPL; ++i) {
     const int c = 4 * (lane + 32 * i);
     float sh[4], sc[4];
-    load4_bf16(mr + shift_off + c, sh);
-    load4_bf16(mr + scale_off + c, sc);
+    unpack4_bf16(shp[i], sh);
+    unpack4_bf16(scp[i], sc);
     const float o0 = fmaf((v[i].x - mean) * rstd, 1.f + sc[0], sh[0]);
     const float o1 = fmaf((v[i].y - mean) * rstd, 1.f + sc[1], sh[1]);
     const float o2 = fmaf((v[i].z - mean) * rstd, 1.f + sc[2], sh[2]);
