@@ -192,7 +192,7 @@ struct StepConst {
 // sampler update of x[m]. With `eval_out` the raw outputs of both rows are
 // written there instead and x is left alone.
 constexpr int FIN_THREADS = 256;
-__global__ void __launch_bounds__(FIN_THREADS) final_kernel(const float* __restrict__ xh, const bf16* __restrict__ mod,
+__global__ void __launch_bounds__(FIN_THREADS, 2) final_kernel(const float* __restrict__ xh, const bf16* __restrict__ mod,
                                                             int ldm, int shift_off, int scale_off,
                                                             const bf16* __restrict__ wout, const float* __restrict__ bout,
                                                             int M, int w, int td, float eps, StepConst sc,
@@ -209,36 +209,46 @@ __global__ void __launch_bounds__(FIN_THREADS) final_kernel(const float* __restr
   if (m >= M) return;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int NW = FIN_THREADS / 32;
-  for (int s = 0; s < 2; ++s) {
-    const int r = s == 0 ? m : M + m;
+  // both rows at once: threads 0-127 normalise row m (conditional), threads
+  // 128-255 row M + m (unconditional); each thread holds w / 128 <= 16
+  // columns t + 128 i, and the modulation loads go out with the row's
+  {
+    static_assert(FIN_THREADS == 256, "two rows of 128 threads");
+    const int g = tid >> 7, t = tid & 127;
+    const int r = g == 0 ? m : M + m;
+    const int n = w >> 7;
     const float* xr = xh + (size_t)r * w;
+    const bf16* mr = mod + (size_t)r * ldm;
+    float v[16], sh[16], scl[16];
     float sum = 0.f;
-    for (int c = tid; c < w; c += FIN_THREADS) {
-      const float a = xr[c];
-      h[s * w + c] = a;
-      sum += a;
-    }
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if (i < n) {
+        const int c = t + 128 * i;
+        sh[i] = to_f(mr[shift_off + c]);
+        scl[i] = to_f(mr[scale_off + c]);
+        v[i] = xr[c];
+        sum += v[i];
+      }
     sum = warp_sum(sum);
     if (lane == 0) red[warp] = sum;
     __syncthreads();
-    float tot = 0.f;
-    for (int k = 0; k < NW; ++k) tot += red[k];
-    const float mean = tot / (float)w;
+    const float mean = ((red[4 * g] + red[4 * g + 1]) + (red[4 * g + 2] + red[4 * g + 3])) / (float)w;
     float q = 0.f;
-    for (int c = tid; c < w; c += FIN_THREADS) {
-      const float d = h[s * w + c] - mean;
-      q += d * d;
-    }
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if (i < n) {
+        const float d = v[i] - mean;
+        q = fmaf(d, d, q);
+      }
     q = warp_sum(q);
-    __syncthreads();  // every thread has read red[] for the mean
-    if (lane == 0) red[warp] = q;
+    if (lane == 0) red[NW + warp] = q;
     __syncthreads();
-    float qt = 0.f;
-    for (int k = 0; k < NW; ++k) qt += red[k];
+    const float qt = (red[NW + 4 * g] + red[NW + 4 * g + 1]) + (red[NW + 4 * g + 2] + red[NW + 4 * g + 3]);
     const float rstd = rsqrtf(qt / (float)w + eps);
-    const bf16* mr = mod + (size_t)r * ldm;
-    for (int c = tid; c < w; c += FIN_THREADS)
-      h[s * w + c] = fmaf((h[s * w + c] - mean) * rstd, 1.f + to_f(mr[scale_off + c]), to_f(mr[shift_off + c]));
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if (i < n) h[g * w + t + 128 * i] = fmaf((v[i] - mean) * rstd, 1.f + scl[i], sh[i]);
     __syncthreads();
   }
   // 2 rows x 2 td outputs, one warp per output at a time; each lane takes 8
