@@ -107,7 +107,8 @@ constexpr bool is_bf16out() { return EK == BF16OUT || EK == BF16OUT_SILU; }
 template <int BN, int EK, int BK>
 struct Cfg {
   static constexpr int ATOMS = BK / ATOM_K;
-  static constexpr int STAGES = BK == 128 ? (is_wide<EK>() ? 2 : 3)
+  // (64-wide tiles, with half the B tile per stage, afford one more stage)
+  static constexpr int STAGES = BK == 128 ? (is_wide<EK>() ? 2 : 3) + (BN == 64 ? 1 : 0)
                                           : is_wide<EK>() ? (BN == 256 ? 3 : BN == 192 ? 4 : 5)
                                                              : (BN == 256 ? 4 : BN == 192 ? 5 : 6);
   static constexpr uint32_t A_BYTES = BM * BK * 2;
