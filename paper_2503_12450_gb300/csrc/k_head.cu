@@ -376,6 +376,7 @@ namespace {
 
 template <class F>
 lazymar_status hlaunch(lazymar_head* h, double flops, const char* what, F&& f) {
+  NvtxRange range(what);
   cudaError_t e = f();
   if (e != cudaSuccess) return head_cuda(e, what);
   h->launches += 1;
@@ -753,6 +754,7 @@ lazymar_status stage(lazymar_head* h, cudaStream_t st, const int32_t* pos, int M
 extern "C" lazymar_status lazymar_head_sample(lazymar_head* h, const void* z, int B, int n_img, const int32_t* pos,
                                               int n_new, const float* noise, float gamma, float temperature,
                                               float* x_out, void* stream) {
+  NvtxRange range("lazymar_head_sample");
   HD_TRY(check_call(h, z, B, n_img, pos, n_new));
   if (!noise || !x_out) return head_fail(LAZYMAR_ERR_INVALID_ARG, "NULL noise or x_out");
   HeadGuard g(h->dev);

@@ -167,6 +167,7 @@ struct DeviceGuard {
 template <class F>
 lazymar_status launch(lazymar_handle* h, int cls, double flops, double bytes, cudaStream_t st, const char* what,
                       F&& f) {
+  NvtxRange range(what);
   lazymar_handle::Ev* ev = nullptr;
   if (h && h->profiling) {
     if (h->ev_used == h->evs.size()) {
@@ -612,6 +613,7 @@ lazymar_status run_body(lazymar_handle* h, cudaStream_t st, const lazymar_handle
 
 extern "C" lazymar_status lazymar_full_step(lazymar_handle* h, const lazymar_step_in* in, float gamma, void* z_out,
                                             void* guided_out, void* stream) {
+  NvtxRange range("lazymar_full_step");
   LM_TRY(check_step_in(h, in));
   DeviceGuard dg(h->dev);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -633,6 +635,7 @@ extern "C" lazymar_status lazymar_full_step(lazymar_handle* h, const lazymar_ste
 extern "C" lazymar_status lazymar_cached_step(lazymar_handle* h, const lazymar_step_in* in, int n_compute,
                                               int use_cond_cache, float gamma, const int32_t* idx_in,
                                               int32_t* idx_out, void* z_out, void* guided_out, void* stream) {
+  NvtxRange range(use_cond_cache ? "lazymar_cached_step (condition cache reused)" : "lazymar_cached_step");
   LM_TRY(check_step_in(h, in));
   if (n_compute < 0 || n_compute > h->T) return fail(LAZYMAR_ERR_INVALID_ARG, "n_compute outside 0..T");
   if (!h->primed) return fail(LAZYMAR_ERR_STATE, "cached step before any full step");

@@ -3,6 +3,7 @@
 // mma.sync, ldmatrix) and the launchers each kernel file exports.
 #pragma once
 
+#include <nvtx3/nvToolsExt.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -441,6 +442,15 @@ cudaError_t launch_topk(const Ctx& c, const double* S, int rows, int T, int N, i
 cudaError_t launch_idx_check(const Ctx& c, const int* idx_in, int rows, int T, int N, int* idx, int* row_map);
 cudaError_t launch_cfg(const Ctx& c, int dtype, int mode, const void* zc, const void* zu, void* delta,
                        float gamma, size_t n, void* zu_out, void* g_out);
+
+// NVTX range for the lifetime of the object (header-only NVTX v3: a no-op
+// unless a profiler has attached its tool library).
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 // Records `msg` as the calling thread's last error (lazymar_last_error) and
 // returns `s`.
