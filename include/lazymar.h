@@ -214,8 +214,11 @@ lazymar_status lazymar_select_tokens_ex(int dtype, const void *v_cur, void *v_ca
  * only. The similarity scratch is a fixed array inside the library, holding
  * LAZYMAR_SELECT_NOALLOC_MAX_TOKENS doubles (2 MiB) on every device that loads
  * it, until the process exits; rows * T above that limit returns
- * LAZYMAR_ERR_INVALID_ARG. The first call on a device looks up the array's
- * device address (make that first call before any stream capture). All calls
+ * LAZYMAR_ERR_INVALID_ARG. Every call looks up the array's device address on
+ * the current device (cudaGetSymbolAddress, which allocates nothing), so the
+ * address stays right after a device reset; the first call on a device also
+ * loads the library's device code there, so make it before any stream
+ * capture. All calls
  * share the one array and leave their similarities in it: calls whose work
  * can overlap on the GPU (different streams, or different host threads) race
  * and must be serialised by the caller. No cudaMalloc, cudaFree or other
@@ -279,6 +282,15 @@ lazymar_status lazymar_layernorm(int dtype, const float *x, const int32_t *row_m
  * (k - k0) % tau_cfg != 0. Returns bit 0 = full step, bit 1 = reuse the
  * condition cache, or -1 for invalid arguments. */
 int lazymar_plan_step(int k, int k0, int tau, int tau_cfg, int use_cond_cache);
+
+/* Copies the selection reference of the first `rows` rows, [rows, T, D] in the
+ * handle's dtype, to dst (device or host memory, caller-owned), on `stream`.
+ * The reference is C^{l=3} of Eq. 8: the representation each row had when it
+ * last ran (after a cached step, this step's block s-1 value matrix or
+ * features). Reading it before and after a cached step gives the two inputs
+ * of that step's Eq. 8 selection. Returns STATE before the first full step,
+ * INVALID_ARG for rows outside 1..2 max_batch or a NULL dst. */
+lazymar_status lazymar_read_reference(lazymar_handle *h, int rows, void *dst, void *stream);
 
 /* Step execution. Each step first copies its inputs (latents, mask, labels,
  * idx_in) into handle-owned buffers on `stream`, so the device work reads

@@ -7,8 +7,13 @@
 // norms in fp64. bf16 x bf16 products are exact in fp64, and so are their sums
 // for any realistic dynamic range, which makes S independent of the summation
 // order: the oracle's fp64 sum gives bit-identical S, hence bit-identical
-// selections. The current vector is copied over the cached one (the cache now
-// holds this step's values).
+// selections (similarity_int_kernel computes those sums exactly on the integer
+// pipe). fp32 x fp32 products are exact in fp64 too, but a sum of them is
+// rounded at every addition, so the kernel's lane-strided order and the
+// oracle's pairwise order can differ in the last bits of S (a relative 1e-15
+// or so). Two tokens whose similarities lie that close may then be ordered
+// differently; every other fp32 selection is identical. The current vector is
+// copied over the cached one (the cache now holds this step's values).
 //
 // topk_kernel: one CTA per row. Each token's rank under the strict total order
 // (S ascending, index ascending; NaN counted as -inf) is counted against all T
@@ -16,7 +21,6 @@
 // block-wide ballot/prefix scan writes them in ascending index order together
 // with the gather/scatter row map r*T + t.
 #include <cfloat>
-#include <mutex>
 
 #include "lazymar_internal.cuh"
 
@@ -359,18 +363,14 @@ constexpr int kMaxDevices = 64;
 // On the host, the name g_select_scratch denotes a host-side stand-in, not
 // device memory: handing it to a kernel would fault or, where the GPU can
 // reach host memory, silently use the wrong memory. The device address is
-// looked up once per device, with that device current, and reused.
-static cudaError_t select_scratch(int dev, double** out) {
-  static std::mutex mu;
-  static double* addr[kMaxDevices] = {};
-  std::lock_guard<std::mutex> lock(mu);
-  if (!addr[dev]) {
-    void* p = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&p, g_select_scratch);
-    if (e != cudaSuccess) return e;
-    addr[dev] = static_cast<double*>(p);
-  }
-  *out = addr[dev];
+// looked up on every call, with the caller's device current: the lookup
+// allocates nothing and costs little, and a cached address would go stale
+// when a device reset reloads the module at another address.
+static cudaError_t select_scratch(double** out) {
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_select_scratch);
+  if (e != cudaSuccess) return e;
+  *out = static_cast<double*>(p);
   return cudaSuccess;
 }
 
@@ -407,7 +407,7 @@ extern "C" lazymar_status lazymar_select_tokens_noalloc(int dtype, const void* v
   if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     return report_error(LAZYMAR_ERR_CUDA, "cudaDeviceGetAttribute failed");
   double* S = nullptr;
-  if (select_scratch(dev, &S) != cudaSuccess)
+  if (select_scratch(&S) != cudaSuccess)
     return report_error(LAZYMAR_ERR_CUDA, "cudaGetSymbolAddress of the selection scratch failed");
   // Every S entry the top-N reads is written by the similarity pass of the
   // same call first, so the scratch needs no clearing between calls.

@@ -814,6 +814,16 @@ extern "C" lazymar_status lazymar_sync(lazymar_handle* h, void* stream) {
   return read_error_word(h->err, static_cast<cudaStream_t>(stream));
 }
 
+extern "C" lazymar_status lazymar_read_reference(lazymar_handle* h, int rows, void* dst, void* stream) {
+  if (!h || !dst) return fail(LAZYMAR_ERR_INVALID_ARG, "NULL handle or destination");
+  if (rows < 1 || rows > h->max_rows) return fail(LAZYMAR_ERR_INVALID_ARG, "rows outside 1..2 max_batch");
+  if (!h->primed) return fail(LAZYMAR_ERR_STATE, "no full step has run yet");
+  DeviceGuard dg(h->dev);
+  const size_t bytes = (size_t)rows * h->T * h->D * h->es;
+  LM_CUDA(cudaMemcpyAsync(dst, h->ref, bytes, cudaMemcpyDefault, static_cast<cudaStream_t>(stream)));
+  return LAZYMAR_OK;
+}
+
 extern "C" lazymar_status lazymar_selftest_wait(int limit_us, void* stream) {
   if (limit_us < 1 || limit_us > 1000000) return fail(LAZYMAR_ERR_INVALID_ARG, "limit_us outside 1..1000000");
   Ctx c;

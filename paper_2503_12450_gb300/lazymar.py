@@ -109,6 +109,7 @@ def lib():
         "lazymar_layernorm": (st, [i, vp, vp, vp, vp, vp, i, i, f, vp]),
         "lazymar_plan_step": (i, [i, i, i, i, i]),
         "lazymar_sync": (st, [vp, vp]),
+        "lazymar_read_reference": (st, [vp, i, vp, vp]),
         "lazymar_device_check": (st, [vp]),
         "lazymar_selftest_wait": (st, [i, vp]),
         "lazymar_set_profiling": (st, [vp, i]),
@@ -277,6 +278,10 @@ def lazymar_plan_step(k, k0, tau, tau_cfg, use_cond_cache=True):
 
 def lazymar_sync(h, stream=None):
     _check(lib().lazymar_sync(h.ptr, _stream(stream)))
+
+
+def lazymar_read_reference(h, rows, dst, stream=None):
+    _check(lib().lazymar_read_reference(h.ptr, int(rows), _ptr(dst), _stream(stream)))
 
 
 def lazymar_selftest_wait(limit_us, stream=None):

@@ -133,6 +133,41 @@ def test_select_tokens_exponent_range_and_specials(D):
     assert torch.equal(g_ref.view(torch.int16), g_cur.view(torch.int16))
 
 
+def test_select_tokens_fp32_near_ties():
+    """fp32 similarities are fp64 sums rounded at every addition, in the
+    kernel's order on the GPU and in numpy's on the CPU, so mathematically
+    equal similarities may come out a few ulps apart on either side. Tokens
+    t and t + 32 carry the same vectors with their elements permuted (equal
+    exact sums, different rounding) and the budget N cuts through those
+    pairs. The GPU's selection must be valid against the oracle's S up to
+    8 ulps; every token outside that band is selected exactly as the oracle
+    selects it."""
+    torch = torch_cuda()
+    rows, T, D, N = 4, 64, 256, 40
+    rng = np.random.default_rng(31)
+    ref = rng.standard_normal((rows, T, D)).astype(np.float32)
+    cur = (ref + 0.3 * rng.standard_normal((rows, T, D))).astype(np.float32)
+    perm = rng.permutation(D)
+    cur[:, 32:], ref[:, 32:] = cur[:, :32][:, :, perm], ref[:, :32][:, :, perm]
+    g_cur, g_ref = dev(cur), dev(ref)
+    idx = torch.full((rows, N), -1, dtype=torch.int32, device="cuda")
+    lm.lazymar_select_tokens(DT["fp32"], g_cur, g_ref, rows, T, D, N, idx)
+    sync()
+    got = idx.cpu().numpy()
+    for r in range(rows):
+        S = O.cosine_similarity(cur[r], ref[r])
+        margin = 8 * np.spacing(np.abs(S).max())
+        sel = set(got[r].tolist())
+        assert len(sel) == N and got[r].tolist() == sorted(sel)
+        for a in sel:
+            for b in set(range(T)) - sel:
+                assert S[a] <= S[b] + margin, (r, a, b)
+        thr = np.sort(S)[N - 1]
+        clear = np.abs(S - thr) > margin
+        expect = set(O.select_compute(S, N).tolist())
+        assert {t for t in range(T) if clear[t] and t in sel} == {t for t in range(T) if clear[t] and t in expect}
+
+
 # --------------------------------------------------------------------------
 # Condition cache / guidance (Eq. 7 reading, Eq. 10)
 # --------------------------------------------------------------------------

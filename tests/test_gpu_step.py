@@ -8,12 +8,16 @@ GPU's own similarity selection bit-exact.
 bf16 (MAR-B/L/H, high resolution): the GPU runs the full batch in the launch
 configuration the benchmark times; the oracle recomputes sampled cond/uncond
 pairs (rows are independent). bf16 arithmetic moves the similarities of
-near-tied tokens, so the GPU's own selection is checked for validity (every
-token the oracle finds clearly changed is selected, none it finds clearly
-unchanged is) and the features are compared with both sides running the
-oracle's I_compute (passed in through idx_in): within 2e-2 and per-token
-cosine >= 0.999. The guided output u + gamma (c - u) is a linear map of the
-features and gets that tolerance propagated through it (see _gpu.guided_ok).
+near-tied tokens, so the two sides need not pick the same tokens. What is
+unique is checked exactly: the GPU's selection equals Eq. 8's rule applied to
+the GPU's own block s-1 value matrices (read back before and after the step),
+bit for bit, in every row. Those value matrices match the oracle's within the
+bf16 tolerance, and the selection is valid against the oracle's similarities
+(every token the oracle finds clearly changed is selected, none it finds
+clearly unchanged is). Features are compared with both sides running the same
+I_compute: within 2e-2 and per-token cosine >= 0.999. The guided output
+u + gamma (c - u) is a linear map of the features and gets that tolerance
+propagated through it (see _gpu.guided_ok).
 """
 import numpy as np
 import pytest
@@ -66,6 +70,13 @@ class Run:
                                select_keys=None if keys is None else dev_int(keys.view(np.int32)))
         lm.lazymar_sync(self.h)
         return host(z), host(g), idx.cpu().numpy()[:, :n]
+
+    def reference(self, rows):
+        """The handle's selection reference of the first `rows` rows, as fp64."""
+        t = empty((rows, self.T, self.D), self.dtype)
+        lm.lazymar_read_reference(self.h, rows, t)
+        lm.lazymar_sync(self.h)
+        return host(t)
 
     def oracle_pair(self, b):
         return O.Cache(self.cfg, 1), (slice(b, b + 1))
@@ -267,6 +278,14 @@ def test_step_state_and_device_errors():
 # bf16 configurations at full batch, sampled pairs against the oracle
 # --------------------------------------------------------------------------
 
+def check_own_selection(I_gpu, ref_before, ref_after, N):
+    """Eq. 8 on the GPU's own value matrices: cosine of this step's values and
+    the previous ones, the N least similar tokens, bit for bit in every row."""
+    S = O.cosine_similarity(ref_after, ref_before)
+    for r in range(I_gpu.shape[0]):
+        assert I_gpu[r].tolist() == O.select_compute(S[r], N).tolist(), r
+
+
 def check_selection(gpu_rows, S_ref, N):
     """The GPU's own selection agrees with the oracle wherever the oracle's
     similarities are clearly separated from the selection threshold."""
@@ -293,7 +312,10 @@ def run_bf16(name, pairs, reuse, n_before=100, n_after=104):
     N = synth.n_compute(cfg)
 
     z0g, g0g = r.full(st0)
+    ref0 = r.reference(2 * B)
     _, _, I_own = r.cached(st1, N, False)
+    ref1 = r.reference(2 * B)
+    check_own_selection(I_own, ref0, ref1, N)
     r.full(st0)
 
     report = {}
@@ -307,6 +329,8 @@ def run_bf16(name, pairs, reuse, n_before=100, n_after=104):
         assert min_cos(z0g[rows], z0) >= COS_MIN
         z1, g1, I1, S1 = O.cached_step(cfg, r.W, c, st1[0][sl], st1[1][sl], r.labels[sl], N, False, GAMMA)
         report[b] = check_selection(I_own[rows], S1, N)
+        # the GPU's block s-1 value matrices of the pair against the oracle's
+        assert max_rel(ref1[rows], c.ref) < TOL["bf16"] and min_cos(ref1[rows], c.ref) >= COS_MIN
         refs[b] = (c, z1, g1, I1)
 
     forced = I_own.copy()
@@ -357,6 +381,91 @@ def test_mar_h_steps():
 def test_hires_steps():
     rep = run_bf16("hires", pairs=[3], reuse=False, n_before=400)
     print("high-resolution selection overlap with the oracle:", rep)
+
+
+def schedule_inputs(cfg):
+    """Latents and masks of every decoding step of the cosine mask schedule."""
+    order, table = synth.make_order(cfg), synth.make_latent_table(cfg)
+    m = synth.mask_counts(cfg["steps"], cfg["n_img"])
+    return [synth.step_state(cfg, order, table, cfg["n_img"] - (m[k - 1] if k > 0 else cfg["n_img"]))
+            for k in range(cfg["steps"])]
+
+
+@pytest.mark.parametrize("tau_cfg", [2, 3])
+def test_tiny_whole_schedule_matches_oracle(tau_cfg):
+    """The tiny fp32 model through all 64 decoding steps (k0 = 4, tau = 9): full
+    steps, cached steps with both pathways and condition-reuse steps, in every
+    order the schedule produces (tau_cfg = 2: reuse -> both -> reuse; tau_cfg =
+    3 adds reuse -> reuse; cached -> full every 9 steps). Each step: the
+    selection bit-exact against the oracle's own (and against Eq. 8 on the
+    GPU's own value matrices), final features and guided output within 1e-4.
+    The unconditional rows of a reuse step do not run, so the next step with
+    both pathways compares them against values two or more steps old; both
+    sides must carry that state alike."""
+    r = Run("tiny", tau_cfg=tau_cfg)
+    cfg = r.cfg
+    N = synth.n_compute(cfg)
+    c = O.Cache(cfg, 1)
+    kinds = []
+    for k, (lat, m) in enumerate(schedule_inputs(cfg)):
+        full, reuse = O.plan(k, cfg["k0"], cfg["tau"], tau_cfg)
+        assert lm.lazymar_plan_step(k, cfg["k0"], cfg["tau"], tau_cfg) == (full, reuse)
+        if full:
+            z, g = O.full_step(cfg, r.W, c, lat, m, r.labels, GAMMA)
+            zg, gg = r.full((lat, m))
+        else:
+            rows = 1 if reuse else 2
+            before = r.reference(rows)
+            z, g, I, _ = O.cached_step(cfg, r.W, c, lat, m, r.labels, N, reuse, GAMMA)
+            zg, gg, Ig = r.cached((lat, m), N, reuse)
+            check_own_selection(Ig, before, r.reference(rows), N)
+            assert Ig.tolist() == I.tolist(), k
+        assert max_rel(zg, z) < TOL["fp32"] and max_rel(gg, g) < TOL["fp32"], k
+        assert min_cos(zg, z) >= COS_MIN, k
+        kinds.append("F" if full else ("R" if reuse else "C"))
+    seq = "".join(kinds)
+    assert "RC" in seq and "CR" in seq and "RF" in seq
+    assert ("RR" in seq) == (tau_cfg == 3)
+    r.h.close()
+
+
+def test_mar_b_schedule_prefix_matches_oracle():
+    """The first 12 decoding steps of the MAR-B schedule (5 full, then cached
+    steps alternating condition reuse and both pathways) at full batch, bf16.
+    The GPU selects on its own every step; the oracle follows the GPU's
+    selection for one sampled pair, so the two caches describe the same
+    decode. Each cached step: the selection bit-exact against Eq. 8 on the
+    GPU's own value matrices, valid against the oracle's similarities, and the
+    features of the pair within the bf16 tolerance."""
+    r = Run("mar_b")
+    cfg, B = r.cfg, r.B
+    N = synth.n_compute(cfg)
+    b = 7
+    rows_b = pair_rows(B, b)
+    sl = slice(b, b + 1)
+    c = O.Cache(cfg, 1)
+    overlaps = []
+    for k, (lat, m) in enumerate(schedule_inputs(cfg)[:12]):
+        full, reuse = O.plan(k, cfg["k0"], cfg["tau"], cfg["tau_cfg"])
+        if full:
+            zg, gg = r.full((lat, m))
+            z, g = O.full_step(cfg, r.W, c, lat[sl], m[sl], r.labels[sl], GAMMA)
+        else:
+            rows = B if reuse else 2 * B
+            before = r.reference(rows)
+            zg, gg, Ig = r.cached((lat, m), N, reuse)
+            after = r.reference(rows)
+            check_own_selection(Ig, before, after, N)
+            pr = [b] if reuse else rows_b
+            z, g, I, S = O.cached_step(cfg, r.W, c, lat[sl], m[sl], r.labels[sl], N, reuse, GAMMA, idx=Ig[pr])
+            overlaps += check_selection(Ig[pr], S, N)
+            assert max_rel(after[pr], c.ref[:len(pr)]) < TOL["bf16"], k
+        assert max_rel(zg[rows_b], z) < TOL["bf16"], k
+        assert min_cos(zg[rows_b], z) >= COS_MIN, k
+        assert guided_ok(gg[b], g[0], z, GAMMA, TOL["bf16"]), k
+    print("MAR-B prefix: selection overlap with the oracle's own choice per cached row:",
+          [round(o, 2) for o in overlaps])
+    r.h.close()
 
 
 def test_graph_replay_matches_eager_execution():

@@ -41,6 +41,27 @@ def test_noalloc_selection_matches_allocating_entry_point_on_two_calls():
         assert torch.equal(a_ref, b_ref) and torch.equal(b_ref, b_cur)
 
 
+# fp32 inputs; no token recomputed; T = 8192, where the top-N's key array
+# (64 KiB) needs the opt-in shared-memory size; rows x T at the limit.
+MORE_CASES = [(2, 80, 256, 20, "fp32", 903), (3, 320, 768, 0, "bf16", 904), (16, 8192, 64, 1000, "bf16", 905),
+              (256, 1024, 8, 100, "bf16", 906)]
+
+
+@pytest.mark.parametrize("rows,T,D,N,dtype,seed", MORE_CASES)
+def test_noalloc_selection_more_shapes(rows, T, D, N, dtype, seed):
+    torch = torch_cuda()
+    cur, ref = synth.similarity_inputs(rows, T, D, seed=seed, dtype=dtype)
+    a_cur, a_ref = dev(cur, dtype), dev(ref, dtype)
+    b_cur, b_ref = dev(cur, dtype), dev(ref, dtype)
+    idx_a = torch.full((rows, max(N, 1)), -1, dtype=torch.int32, device="cuda")
+    idx_b = torch.full((rows, max(N, 1)), -2, dtype=torch.int32, device="cuda")
+    lm.lazymar_select_tokens(DT[dtype], a_cur, a_ref, rows, T, D, N, idx_a)
+    lm.lazymar_select_tokens_noalloc(DT[dtype], b_cur, b_ref, rows, T, D, N, idx_b)
+    sync()
+    assert torch.equal(idx_a[:, :N], idx_b[:, :N])
+    assert torch.equal(a_ref, b_ref) and torch.equal(b_ref, b_cur)
+
+
 def test_noalloc_rejects_sizes_beyond_its_scratch():
     torch_cuda()
     # 257 rows x 1024 tokens = 263,168 > LAZYMAR_SELECT_NOALLOC_MAX_TOKENS (262,144);
