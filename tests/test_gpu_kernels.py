@@ -266,19 +266,26 @@ def test_linear_fp32(M, N, K, epi):
 # Attention (Eq. 3 with a query subset)
 # --------------------------------------------------------------------------
 
-@pytest.mark.parametrize("rows,n_q,T,heads,dh,dtype", [
-    (2, 50, 320, 12, 64, "bf16"),    # MAR-B cached layer
-    (2, 320, 320, 4, 64, "bf16"),    # full layer
-    (1, 272, 1088, 2, 64, "bf16"),   # high resolution cached layer
-    (3, 50, 320, 4, 80, "bf16"),     # MAR-H head width
-    (2, 65, 130, 2, 80, "bf16"),     # ragged queries and keys
-    (1, 1, 1, 1, 64, "bf16"),
-    (2, 20, 80, 4, 64, "fp32"),      # tiny
-    (1, 3, 5, 2, 32, "fp32"),
+@pytest.mark.parametrize("rows,n_q,T,heads,dh,dtype,q_std", [
+    (2, 50, 320, 12, 64, "bf16", 1.0),    # MAR-B cached layer
+    (2, 320, 320, 4, 64, "bf16", 1.0),    # full layer
+    (1, 272, 1088, 2, 64, "bf16", 1.0),   # high resolution cached layer
+    (3, 50, 320, 4, 80, "bf16", 1.0),     # MAR-H head width, cached layer
+    (2, 320, 320, 16, 80, "bf16", 1.0),   # MAR-H full layer (three query tiles)
+    (2, 65, 130, 2, 80, "bf16", 1.0),     # ragged queries and keys
+    (1, 129, 200, 3, 80, "bf16", 1.0),    # one query past a tile, a ragged key chunk
+    (1, 1, 1, 1, 80, "bf16", 1.0),
+    (1, 1, 1, 1, 64, "bf16", 1.0),
+    # scores of std ~6 (log2 units): the running maximum is raised mid-row
+    # and O in tensor memory rescaled
+    (2, 50, 320, 4, 64, "bf16", 4.0),
+    (2, 50, 320, 4, 80, "bf16", 4.0),
+    (2, 20, 80, 4, 64, "fp32", 1.0),      # tiny
+    (1, 3, 5, 2, 32, "fp32", 1.0),
 ])
-def test_attention(rows, n_q, T, heads, dh, dtype):
+def test_attention(rows, n_q, T, heads, dh, dtype, q_std):
     D = heads * dh
-    q = synth.tensor((rows, n_q, D), 21, dtype=dtype)
+    q = synth.tensor((rows, n_q, D), 21, std=q_std, dtype=dtype)
     k = synth.tensor((rows, T, D), 22, dtype=dtype)
     v = synth.tensor((rows, T, D), 23, dtype=dtype)
     o = empty((rows, n_q, D), dtype)
