@@ -299,7 +299,10 @@ lazymar_status lazymar_read_reference(lazymar_handle *h, int rows, void *dst, vo
  * combination is seen, is captured into a CUDA graph the second time and
  * replayed from then on; the CFG combine and the output copies are launched
  * after it, so gamma may change from call to call. enable = 0 runs every step
- * eagerly. Graphs are never used while profiling is on. */
+ * eagerly. While profiling is on, each combination is captured on its first
+ * use together with an event record around every launch, into a graph of its
+ * own, and replayed; the per-kernel times are then device times, free of the
+ * host's launch submission. */
 lazymar_status lazymar_set_graphs(lazymar_handle *h, int enable);
 
 /* Waits for `stream`, then reports (and clears) errors the handle's kernels

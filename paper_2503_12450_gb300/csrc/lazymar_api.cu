@@ -140,8 +140,15 @@ struct lazymar_handle {
     cudaGraphExec_t exec = nullptr;
     int eager_runs = 0;
     lazymar_stats delta{};
+    std::vector<Ev> evs;   // profiled graphs: the event pairs recorded by its nodes
+    bool pending = false;  // profiled graphs: replayed, events not read yet
   };
   std::map<GraphKey, GraphEntry> graphs;
+  // Profiled step bodies: captured with an event record around every launch,
+  // so that per-kernel times are device times and exclude the host's launch
+  // submission (eagerly issued launches can leave the GPU idle between the
+  // events of a short kernel).
+  std::map<GraphKey, GraphEntry> pgraphs;
   bool use_graphs = true;
   cudaStream_t gstream = nullptr;  // capture / replay stream
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
@@ -169,6 +176,7 @@ lazymar_status launch(lazymar_handle* h, int cls, double flops, double bytes, cu
                       F&& f) {
   NvtxRange range(what);
   lazymar_handle::Ev* ev = nullptr;
+  unsigned ev_flags = cudaEventRecordDefault;
   if (h && h->profiling) {
     if (h->ev_used == h->evs.size()) {
       lazymar_handle::Ev e{};
@@ -178,10 +186,19 @@ lazymar_status launch(lazymar_handle* h, int cls, double flops, double bytes, cu
     }
     ev = &h->evs[h->ev_used++];
     ev->cls = cls;
-    LM_CUDA(cudaEventRecord(ev->a, st));
+    // under stream capture the records must be external to become
+    // event-record nodes of the graph (a plain record would only mark a
+    // capture dependency)
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    LM_CUDA(cudaStreamIsCapturing(st, &cs));
+    ev_flags = cs == cudaStreamCaptureStatusActive ? cudaEventRecordExternal : cudaEventRecordDefault;
+    LM_CUDA(cudaEventRecordWithFlags(ev->a, st, ev_flags));
   }
   cudaError_t e = f();
-  if (ev) LM_CUDA(cudaEventRecord(ev->b, st));
+  if (ev) {
+    const cudaError_t eb = cudaEventRecordWithFlags(ev->b, st, ev_flags);
+    if (eb != cudaSuccess) return cuda_fail(eb, "event record after a launch");
+  }
   if (e != cudaSuccess) return cuda_fail(e, what);
   if (h) {
     lazymar_kernel_stats& k = h->stats.k[cls];
@@ -376,6 +393,13 @@ extern "C" void lazymar_destroy(lazymar_handle* h) {
   DeviceGuard g(h->dev);
   for (auto& kv : h->graphs)
     if (kv.second.exec) cudaGraphExecDestroy(kv.second.exec);
+  for (auto& kv : h->pgraphs) {
+    if (kv.second.exec) cudaGraphExecDestroy(kv.second.exec);
+    for (auto& e : kv.second.evs) {
+      cudaEventDestroy(e.a);
+      cudaEventDestroy(e.b);
+    }
+  }
   if (h->ev_fork) cudaEventDestroy(h->ev_fork);
   if (h->ev_join) cudaEventDestroy(h->ev_join);
   if (h->gstream) cudaStreamDestroy(h->gstream);
@@ -567,25 +591,49 @@ void add_stats(lazymar_stats& a, const lazymar_stats& d, double sign) {
   }
 }
 
+// Reads the event pairs of a replayed profiled graph into the statistics.
+lazymar_status drain_profiled(lazymar_handle* h, lazymar_handle::GraphEntry& ge) {
+  if (!ge.pending) return LAZYMAR_OK;
+  ge.pending = false;
+  if (ge.evs.empty()) return LAZYMAR_OK;
+  LM_CUDA(cudaEventSynchronize(ge.evs.back().b));
+  for (const auto& e : ge.evs) {
+    float ms = 0.f;
+    LM_CUDA(cudaEventElapsedTime(&ms, e.a, e.b));
+    h->stats.k[e.cls].ms += ms;
+    h->stats.k[e.cls].timed_launches += 1;
+  }
+  return LAZYMAR_OK;
+}
+
 // Runs a step body: eagerly on the caller's stream on its first use (and
-// always while profiling or with graphs disabled); from then on as a CUDA
-// graph, captured on the second use and replayed afterwards. Capture and
-// replay run on the handle's own stream, joined to the caller's stream by
-// events (the legacy default stream cannot be captured).
+// always with graphs disabled); from then on as a CUDA graph, captured on the
+// second use and replayed afterwards. Capture and replay run on the handle's
+// own stream, joined to the caller's stream by events (the legacy default
+// stream cannot be captured). While profiling, the body is captured with its
+// per-launch events into a separate graph on its first use and replayed from
+// there (the events are read by lazymar_get_stats, or before the same graph
+// is replayed again).
 template <class F>
 lazymar_status run_body(lazymar_handle* h, cudaStream_t st, const lazymar_handle::GraphKey& key, F&& body) {
-  if (h->profiling || !h->use_graphs) return body(Ctx{st, h->err, h->num_sms});
-  lazymar_handle::GraphEntry& ge = h->graphs[key];
-  if (!ge.exec && ge.eager_runs++ == 0) return body(Ctx{st, h->err, h->num_sms});
+  if (!h->use_graphs) return body(Ctx{st, h->err, h->num_sms});
+  lazymar_handle::GraphEntry& ge = h->profiling ? h->pgraphs[key] : h->graphs[key];
+  if (!h->profiling && !ge.exec && ge.eager_runs++ == 0) return body(Ctx{st, h->err, h->num_sms});
+  LM_TRY(drain_profiled(h, ge));
   cudaStream_t gs = h->gstream;
   LM_CUDA(cudaEventRecord(h->ev_fork, st));
   LM_CUDA(cudaStreamWaitEvent(gs, h->ev_fork, 0));
   if (!ge.exec) {
     const lazymar_stats before = h->stats;
+    const size_t ev_base = h->ev_used;
     LM_CUDA(cudaStreamBeginCapture(gs, cudaStreamCaptureModeThreadLocal));
     const lazymar_status s = body(Ctx{gs, h->err, h->num_sms});
     cudaGraph_t g = nullptr;
     const cudaError_t e = cudaStreamEndCapture(gs, &g);
+    // events recorded by the captured launches belong to the graph
+    ge.evs.assign(h->evs.begin() + ev_base, h->evs.begin() + h->ev_used);
+    h->evs.erase(h->evs.begin() + ev_base, h->evs.begin() + h->ev_used);
+    h->ev_used = ev_base;
     if (s != LAZYMAR_OK || e != cudaSuccess) {
       if (g) cudaGraphDestroy(g);
       h->stats = before;
@@ -606,6 +654,7 @@ lazymar_status run_body(lazymar_handle* h, cudaStream_t st, const lazymar_handle
   LM_CUDA(cudaEventRecord(h->ev_join, gs));
   LM_CUDA(cudaStreamWaitEvent(st, h->ev_join, 0));
   add_stats(h->stats, ge.delta, 1.0);
+  ge.pending = h->profiling;
   return LAZYMAR_OK;
 }
 
@@ -847,6 +896,7 @@ extern "C" lazymar_status lazymar_set_profiling(lazymar_handle* h, int enable) {
 extern "C" lazymar_status lazymar_get_stats(lazymar_handle* h, lazymar_stats* out) {
   if (!h || !out) return fail(LAZYMAR_ERR_INVALID_ARG, "NULL argument");
   DeviceGuard dg(h->dev);
+  for (auto& kv : h->pgraphs) LM_TRY(drain_profiled(h, kv.second));
   if (h->ev_used > 0) {
     LM_CUDA(cudaEventSynchronize(h->evs[h->ev_used - 1].b));
     for (size_t i = 0; i < h->ev_used; ++i) {

@@ -468,6 +468,32 @@ def test_mar_b_schedule_prefix_matches_oracle():
     r.h.close()
 
 
+def test_profiling_times_every_launch_and_changes_no_result():
+    """With profiling on, step bodies run from graphs that carry an event pair
+    around every launch: the outputs are bit-identical to unprofiled steps and
+    every launch of the profiled steps has a device time."""
+    r = Run("mar_b", batch=2)
+    N = synth.n_compute(r.cfg)
+    sts = [r.state(n) for n in (100, 104, 108)]
+
+    def seq():
+        return [r.full(sts[0]), r.cached(sts[1], N, False), r.cached(sts[2], N, True)]
+    plain = seq()
+    lm.lazymar_set_profiling(r.h, True)
+    lm.lazymar_reset_stats(r.h)
+    for _ in range(2):                      # capture, then replay
+        prof = seq()
+        for a, b in zip(plain, prof):
+            for x, y in zip(a, b):
+                assert np.array_equal(x, y)
+    st = lm.lazymar_get_stats(r.h)
+    lm.lazymar_set_profiling(r.h, False)
+    for name in ("gemm", "attention", "layernorm", "select", "embed"):
+        assert st[name]["launches"] > 0 and st[name]["timed_launches"] == st[name]["launches"], name
+        assert st[name]["ms"] > 0, name
+    r.h.close()
+
+
 def test_graph_replay_matches_eager_execution():
     """Step bodies replayed from CUDA graphs give the same bits as eager launches,
     and a changed gamma is honoured on a replayed step."""
