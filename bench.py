@@ -537,6 +537,20 @@ def profile_case(args, cfg):
                     o = torch.empty(M, n, device=dev, dtype=torch.bfloat16)
                     lm.lazymar_linear(lm.LAZYMAR_BF16, epi, a, w, b, M, n, k, o, n)
                 torch.cuda.synchronize()
+    elif args.profile_case == "steps":
+        # one full and one cached step (both pathways) of the configuration,
+        # every kernel launched eagerly
+        B = cfg["batch"]
+        W = synth.make_weights(cfg)
+        h = lm.lazymar_create(dict(cfg, max_batch=B), W)
+        lm.lazymar_set_graphs(h, False)
+        lat, mask, labels = decode_inputs(cfg, 0)
+        lat, mask, labels = (torch.from_numpy(x).cuda() for x in (lat, mask, labels))
+        g = torch.empty((B, cfg["n_img"], D), device=dev, dtype=torch.bfloat16)
+        lm.lazymar_full_step(h, lat[10], mask[10], labels, B, GAMMA, None, g)
+        lm.lazymar_cached_step(h, lat[11], mask[11], labels, B, N, False, GAMMA, None, None, None, g)
+        lm.lazymar_sync(h)
+        h.close()
     elif args.profile_case == "head":
         B, n_img, td = cfg["batch"], cfg["n_img"], cfg["token_dim"]
         hc = synth.head_config(HEAD_FOR[cfg["name"]])
@@ -633,7 +647,7 @@ def main():
     ap.add_argument("--no-head", action="store_true", help="skip the decode with the diffusion head")
     ap.add_argument("--select", default="least_similar", choices=sorted(SELECT_RULES),
                     help="token-selection strategy of the cached steps (Table 3; default: LazyMAR's)")
-    ap.add_argument("--profile-case", choices=["gemm_layers", "attention_layers", "head"], default=None,
+    ap.add_argument("--profile-case", choices=["gemm_layers", "attention_layers", "head", "steps"], default=None,
                     help="run each kernel of a layer once at the configuration's shapes (for ncu) and exit")
     args = ap.parse_args()
     cfg = synth.config(args.config)
