@@ -509,9 +509,13 @@ def run_ours(args, cfg):
 def profile_case(args, cfg):
     """One launch of each kernel of a layer at the configuration's shapes, for a
     profiler: `gemm_layers` runs QKV, out-proj, fc1 and fc2 on all rows x T
-    tokens and on the recomputed rows x N tokens; `attention_layers` runs the
+    tokens, on the recomputed rows x N tokens and on the half of them a
+    condition-reuse step runs; `attention_layers` runs the
     recomputed-token and the full-layer attention; `head` runs one eager
-    diffusion-head sampling call (100 steps) for 4 new tokens per pair."""
+    diffusion-head sampling call (100 steps) for 4 new tokens per pair;
+    `steps` runs one full and one cached step eagerly; `launch_floor` times the
+    recomputed-token GEMMs and a minimal kernel inside CUDA graphs, back to
+    back and with an event pair around every launch."""
     import torch
     from paper_2503_12450_gb300 import lazymar as lm
     lm.lib()
@@ -520,7 +524,7 @@ def profile_case(args, cfg):
     N = synth.n_compute(cfg)
     dev = "cuda"
     if args.profile_case == "gemm_layers":
-        for M in (rows * T, rows * N):
+        for M in (rows * T, rows * N, rows * N // 2):
             for n, k, epi in [(3 * D, D, lm.LAZYMAR_EPI_QKV), (D, D, lm.LAZYMAR_EPI_RESIDUAL),
                               (4 * D, D, lm.LAZYMAR_EPI_GELU), (D, 4 * D, lm.LAZYMAR_EPI_RESIDUAL)]:
                 a = torch.randn(M, k, device=dev).bfloat16()
@@ -537,6 +541,72 @@ def profile_case(args, cfg):
                     o = torch.empty(M, n, device=dev, dtype=torch.bfloat16)
                     lm.lazymar_linear(lm.LAZYMAR_BF16, epi, a, w, b, M, n, k, o, n)
                 torch.cuda.synchronize()
+    elif args.profile_case == "launch_floor":
+        # Per-launch device time of the recomputed-token GEMMs (both pathways,
+        # M = rows x N; condition reuse, M = rows x N / 2) and of a minimal
+        # kernel, each launched 20 times inside a CUDA graph: back to back (as
+        # in the decode, consecutive launches overlap through programmatic
+        # dependent launch) and with a CUDA event pair around every launch (how
+        # the benchmark's per-kernel profile times them)
+        R = 20
+
+        def timed_graph(call):
+            call()
+            torch.cuda.synchronize()
+            g1 = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g1, capture_error_mode="relaxed"):
+                for _ in range(R):
+                    call()
+            evs = [(torch.cuda.Event(enable_timing=True, external=True),
+                    torch.cuda.Event(enable_timing=True, external=True)) for _ in range(R)]
+            g2 = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g2, capture_error_mode="relaxed"):
+                for x, y in evs:
+                    x.record()
+                    call()
+                    y.record()
+            for _ in range(3):
+                g1.replay()
+                g2.replay()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            g1.replay()
+            e1.record()
+            torch.cuda.synchronize()
+            back = e0.elapsed_time(e1) / R * 1e3
+            g2.replay()
+            torch.cuda.synchronize()
+            return back, sum(x.elapsed_time(y) for x, y in evs) / R * 1e3
+
+        out = {}
+        zc = torch.randn(8, device=dev).bfloat16()
+        zu, dl, gg = torch.randn_like(zc), torch.empty_like(zc), torch.empty_like(zc)
+        b, e = timed_graph(lambda: lm.lazymar_cfg_combine(lm.LAZYMAR_BF16, lm.LAZYMAR_CFG_REFRESH, zc, zu, dl, GAMMA, 8,
+                                                           None, gg))
+        out["minimal kernel (guidance on 8 elements)"] = {"back_to_back_us": round(b, 2), "events_us": round(e, 2)}
+        for M in (rows * N, rows * N // 2):
+            for name, n, k, epi in [("qkv", 3 * D, D, lm.LAZYMAR_EPI_QKV), ("out", D, D, lm.LAZYMAR_EPI_RESIDUAL),
+                                    ("fc1", 4 * D, D, lm.LAZYMAR_EPI_GELU), ("fc2", D, 4 * D, lm.LAZYMAR_EPI_RESIDUAL)]:
+                a = torch.randn(M, k, device=dev).bfloat16()
+                w = (torch.randn(n, k, device=dev) * 0.05).bfloat16()
+                bias = torch.randn(n, device=dev).bfloat16()
+                if epi == lm.LAZYMAR_EPI_QKV:
+                    q = torch.empty(M, D, device=dev, dtype=torch.bfloat16)
+                    kk, vv = torch.empty_like(q), torch.empty_like(q)
+                    call = lambda: lm.lazymar_linear(lm.LAZYMAR_BF16, epi, a, w, bias, M, n, k, q, D, kk, vv, None)
+                elif epi == lm.LAZYMAR_EPI_RESIDUAL:
+                    o = torch.zeros(M, n, device=dev)
+                    call = lambda: lm.lazymar_linear(lm.LAZYMAR_BF16, epi, a, w, bias, M, n, k, o, n)
+                else:
+                    o = torch.empty(M, n, device=dev, dtype=torch.bfloat16)
+                    call = lambda: lm.lazymar_linear(lm.LAZYMAR_BF16, epi, a, w, bias, M, n, k, o, n)
+                b, e = timed_graph(call)
+                fl = 2.0 * M * n * k
+                out["%s M=%d" % (name, M)] = {"back_to_back_us": round(b, 2), "events_us": round(e, 2),
+                                              "tflops_back_to_back": round(fl / b / 1e6, 1),
+                                              "tflops_events": round(fl / e / 1e6, 1)}
+        print(json.dumps(out, indent=1), flush=True)
     elif args.profile_case == "steps":
         # one full and one cached step (both pathways) of the configuration,
         # every kernel launched eagerly
@@ -647,7 +717,8 @@ def main():
     ap.add_argument("--no-head", action="store_true", help="skip the decode with the diffusion head")
     ap.add_argument("--select", default="least_similar", choices=sorted(SELECT_RULES),
                     help="token-selection strategy of the cached steps (Table 3; default: LazyMAR's)")
-    ap.add_argument("--profile-case", choices=["gemm_layers", "attention_layers", "head", "steps"], default=None,
+    ap.add_argument("--profile-case", choices=["gemm_layers", "attention_layers", "head", "steps", "launch_floor"],
+                    default=None,
                     help="run each kernel of a layer once at the configuration's shapes (for ncu) and exit")
     args = ap.parse_args()
     cfg = synth.config(args.config)
