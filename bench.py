@@ -72,6 +72,7 @@ def workload(cfg, select="least_similar"):
             "cond cache reused on cached steps with (k-k0) %% %d != 0" % cfg["tau_cfg"]),
         "decoding_steps": cfg["steps"],
         "selection": select,
+        "cached_qkv_operands": "e4m3" if cfg.get("qkv_e4m3") else "bf16",
         "l2": "no flush: the per-step working set (%.2f GB weights + %.2f GB K/V cache) exceeds the 129 MB L2" % (
             12 * cfg["depth"] * cfg["width"] ** 2 * 2 / 1e9,
             2 * (cfg["depth"] - cfg["sel_layers"]) * 2 * cfg["batch"] * cfg["T"] * cfg["width"] * 2 / 1e9),
@@ -715,6 +716,8 @@ def main():
     ap.add_argument("--ratio", type=float, default=None, help="recompute ratio (default: the config's)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-head", action="store_true", help="skip the decode with the diffusion head")
+    ap.add_argument("--qkv-e4m3", action="store_true",
+                    help="Q/K/V projection of the cached blocks on 8-bit (E4M3) tensor cores")
     ap.add_argument("--select", default="least_similar", choices=sorted(SELECT_RULES),
                     help="token-selection strategy of the cached steps (Table 3; default: LazyMAR's)")
     ap.add_argument("--profile-case", choices=["gemm_layers", "attention_layers", "head", "steps", "launch_floor"],
@@ -724,6 +727,7 @@ def main():
     cfg = synth.config(args.config)
     if args.ratio is not None:
         cfg["ratio"] = args.ratio
+    cfg["qkv_e4m3"] = 1 if args.qkv_e4m3 else 0
     if args.profile_case:
         profile_case(args, cfg)
     elif args.impl == "reference":

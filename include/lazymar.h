@@ -61,7 +61,7 @@ typedef enum lazymar_status {
   LAZYMAR_ERR_DEVICE = 7        /* a kernel found a bad index or label on the device */
 } lazymar_status;
 
-typedef enum lazymar_dtype { LAZYMAR_F32 = 0, LAZYMAR_BF16 = 1 } lazymar_dtype;
+typedef enum lazymar_dtype { LAZYMAR_F32 = 0, LAZYMAR_BF16 = 1, LAZYMAR_E4M3 = 2 } lazymar_dtype;
 
 /* Which representation of block sel_layers-1 the similarity of Eq. 8 compares:
  * the attention value matrix (Sec. 4.4 "value matrix instead of features";
@@ -107,6 +107,14 @@ typedef struct lazymar_config {
   int criterion;   /* lazymar_criterion */
   float ln_eps;    /* LayerNorm epsilon */
   int select_rule; /* lazymar_select_rule of the cached steps (0 = strategy V) */
+  int qkv_e4m3;    /* 1: the Q/K/V projection of blocks s..L-1 on the recomputed
+                    * tokens runs on 8-bit tensor cores: LN1 output rounded to
+                    * E4M3 (unit scale), W_qkv rounded to E4M3 with one scale
+                    * per output channel (max |w| / 448), fp32 accumulation.
+                    * bf16 only, width % 128 == 0. The paper ran FP16; this is
+                    * an extension, within the bf16 parity tolerance on every
+                    * configuration (E4M3 in the other GEMMs is not: see the
+                    * design notes). 0: bf16 throughout. */
 } lazymar_config;
 
 /* Weights of one pre-LN block, fp32, [out, in] layout (y = x W^T + b).
@@ -264,6 +272,23 @@ lazymar_status lazymar_linear(int dtype, int epilogue, const void *a, const void
                               void *k_out, void *v_out, const int32_t *row_map, int flags,
                               void *stream);
 
+/* lazymar_linear with E4M3 operands (kind::f8f6f4 tensor cores, fp32
+ * accumulation): a [M, K] and w [N, K] hold E4M3 bytes, wscale [N] fp32 the
+ * per-output-column scale of w; y = (a w^T) * wscale + bias (bias bf16, may be
+ * NULL). Epilogues BIAS, GELU (bf16 out) and QKV (bf16 Q/K/V, K/V scattered
+ * through row_map) as for lazymar_linear. K % 128 == 0, N % 128 == 0. The
+ * paper has no 8-bit arithmetic; this is the Q/K/V projection of a
+ * configuration with qkv_e4m3 set. */
+lazymar_status lazymar_linear_e4m3(int epilogue, const void *a, const void *w, const float *wscale,
+                                   const void *bias, int M, int N, int K, void *out, int ldo, void *k_out,
+                                   void *v_out, const int32_t *row_map, int flags, void *stream);
+
+/* E4M3 copy of a bf16 weight matrix w [rows, cols] (cols % 8 == 0) with one
+ * scale per row: scale[r] = max_c |w[r, c]| / 448 (1 for a zero row),
+ * q[r, c] = E4M3(w[r, c] / scale[r]) (nearest, ties to even, saturating).
+ * Device pointers: q [rows, cols] bytes, scale [rows] fp32. */
+lazymar_status lazymar_quantize_e4m3(const void *w, int rows, int cols, void *q, float *scale, void *stream);
+
 /* Multi-head bidirectional attention of Eq. 3 with a query subset: for each row
  * r and head h, O[r, j] = softmax(Q[r, j] K[r]^T / sqrt(dh)) V[r] over all T
  * keys. q, o: [rows, n_q, heads*head_dim]; k, v: [rows, T, heads*head_dim]
@@ -272,7 +297,8 @@ lazymar_status lazymar_attention(int dtype, const void *q, const void *k, const 
                                  int rows, int n_q, int T, int heads, int head_dim, void *stream);
 
 /* LayerNorm over D of fp32 rows: y[m] = LN(x[row_map ? row_map[m] : m]) * g + b,
- * y in dtype, g/b in dtype. D % 128 == 0, D <= 2048. */
+ * y in dtype, g/b in dtype; dtype LAZYMAR_E4M3: g/b bf16, y E4M3 bytes (unit
+ * scale, saturating at 448). D % 128 == 0, D <= 2048. */
 lazymar_status lazymar_layernorm(int dtype, const float *x, const int32_t *row_map, const void *g,
                                  const void *b, void *y, int M, int D, float eps, void *stream);
 

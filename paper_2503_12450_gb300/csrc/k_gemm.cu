@@ -83,7 +83,6 @@ __device__ __forceinline__ void epilogue_apply(const GemmEpi& e, int row, int co
 // ---------------------------------------------------------------------------
 namespace tc {
 constexpr int BM = 128;  // rows per tile = MMA M (one accumulator lane per row)
-constexpr int ATOM_K = 64;  // one 128-byte swizzle atom of bf16 along K (one TMA box)
 
 // Epilogue kinds: BF16OUT stores bf16 (bias / GELU / Q-K-V split); the two
 // residual kinds add into the fp32 residual stream. RESID_WIDE stages whole
@@ -100,19 +99,24 @@ constexpr bool is_wide() { return EK == RESID_WIDE || EK == RESID_WIDE_GATED; }
 template <int EK>
 constexpr bool is_bf16out() { return EK == BF16OUT || EK == BF16OUT_SILU; }
 
-// BK: K per pipeline stage, one or two swizzle atoms. A 128-wide tile runs
-// 128-deep stages (two atoms, eight MMAs per barrier round trip): its
-// 128 x 128 x 16 MMAs are too short to hide the per-stage wait and commit at
-// 64 (measured 13-19 % faster); wider tiles keep 64 for a deeper ring.
-template <int BN, int EK, int BK>
+// BK: K per pipeline stage (elements), one or two swizzle atoms. A 128-wide
+// tile runs 128-deep stages (two atoms, eight MMAs per barrier round trip):
+// its 128 x 128 x 16 MMAs are too short to hide the per-stage wait and commit
+// at 64 (measured 13-19 % faster); wider tiles keep 64 for a deeper ring.
+// F8: E4M3 operands (kind::f8f6f4): a 128-byte atom holds 128 elements and an
+// MMA step is K = 32, still 32 bytes; BK = 128 is one atom, the bytes of a
+// 64-deep bf16 stage.
+template <int BN, int EK, int BK, int F8 = 0>
 struct Cfg {
-  static constexpr int ATOMS = BK / ATOM_K;
+  static constexpr int EB = F8 ? 1 : 2;          // bytes per operand element
+  static constexpr int ATOM_E = 128 / EB;        // elements per 128-byte swizzle atom
+  static constexpr int ATOMS = BK / ATOM_E;
   // (64-wide tiles, with half the B tile per stage, afford one more stage)
-  static constexpr int STAGES = BK == 128 ? (is_wide<EK>() ? 2 : 3) + (BN == 64 ? 1 : 0)
+  static constexpr int STAGES = ATOMS == 2 ? (is_wide<EK>() ? 2 : 3) + (BN == 64 ? 1 : 0)
                                           : is_wide<EK>() ? (BN == 256 ? 3 : BN == 192 ? 4 : 5)
                                                              : (BN == 256 ? 4 : BN == 192 ? 5 : 6);
-  static constexpr uint32_t A_BYTES = BM * BK * 2;
-  static constexpr uint32_t B_BYTES = BN * BK * 2;
+  static constexpr uint32_t A_BYTES = BM * BK * EB;
+  static constexpr uint32_t B_BYTES = BN * BK * EB;
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   // two accumulator buffers (columns [0, BN) and [BN, 2 BN)); the allocation
   // is a power of two
@@ -133,10 +137,11 @@ struct Cfg {
   static constexpr uint32_t STG_PITCH = is_bf16out<EK>() ? 64 : ROW_BYTES + 16;
   static constexpr uint32_t STG_BYTES = 32 * STG_PITCH;
   static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + EPI_WARPS * STG_BYTES + 256;
-  // Instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1),
-  // B bf16 (bits 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
-  static constexpr uint32_t IDESC =
-      (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+  // Instruction descriptor: D fp32 (bit 4); kind::f16 with A and B bf16
+  // (bits 7-9 and 10-12 = 1), or kind::f8f6f4 with A and B E4M3 (format 0);
+  // both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
+  static constexpr uint32_t IDESC = (1u << 4) | (F8 ? 0u : (1u << 7) | (1u << 10)) | ((uint32_t)(BN >> 3) << 17) |
+                                    ((uint32_t)(BM >> 4) << 24);
 };
 
 // Shared-memory matrix descriptor of a K-major tile written by TMA with
@@ -167,14 +172,15 @@ __device__ __forceinline__ bf16* out_row(const GemmEpi& e, int row, int col) {
 }
 }  // namespace tc
 
-template <int BN, int EK, int BK>
-__global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
+template <int BN, int EK, int BK, int F8 = 0>
+__global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
     gemm_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                         const __grid_constant__ CUtensorMap tmO0, const __grid_constant__ CUtensorMap tmO1,
                         const __grid_constant__ CUtensorMap tmO2, int tma_out, int M, int N, int K, GemmEpi epi,
                         unsigned* err) {
-  using C = tc::Cfg<BN, EK, BK>;
+  using C = tc::Cfg<BN, EK, BK, F8>;
   constexpr bool RESID = !tc::is_bf16out<EK>();
+  static_assert(!F8 || EK == tc::BF16OUT, "E4M3 operands: bf16-output epilogue only");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -230,7 +236,7 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
       mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
 #pragma unroll
       for (int a = 0; a < C::ATOMS; ++a)
-        tma_load_2d(&tmB, &full[s], sB + s * C::B_BYTES + a * (C::B_BYTES / C::ATOMS), s * BK + a * tc::ATOM_K, n0);
+        tma_load_2d(&tmB, &full[s], sB + s * C::B_BYTES + a * (C::B_BYTES / C::ATOMS), s * BK + a * C::ATOM_E, n0);
     }
   }
   pdl_wait();
@@ -250,16 +256,16 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
 #pragma unroll
             for (int a = 0; a < C::ATOMS; ++a)
               tma_load_2d(&tmA, &full[stage], sA + stage * C::A_BYTES + a * (C::A_BYTES / C::ATOMS),
-                          kb * BK + a * tc::ATOM_K, m0);
+                          kb * BK + a * C::ATOM_E, m0);
           } else {
             if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
             mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
 #pragma unroll
             for (int a = 0; a < C::ATOMS; ++a) {
               tma_load_2d(&tmA, &full[stage], sA + stage * C::A_BYTES + a * (C::A_BYTES / C::ATOMS),
-                          kb * BK + a * tc::ATOM_K, m0);
+                          kb * BK + a * C::ATOM_E, m0);
               tma_load_2d(&tmB, &full[stage], sB + stage * C::B_BYTES + a * (C::B_BYTES / C::ATOMS),
-                          kb * BK + a * tc::ATOM_K, n0);
+                          kb * BK + a * C::ATOM_E, n0);
             }
           }
           if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
@@ -286,11 +292,14 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
           const uint64_t a0 = tc::sw128_desc(smem_u32(sA + stage * C::A_BYTES));
           const uint64_t b0 = tc::sw128_desc(smem_u32(sB + stage * C::B_BYTES));
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k) {  // +32 bytes per K=16 step inside an atom
-            const int a = k / (tc::ATOM_K / 16), ks = k % (tc::ATOM_K / 16);
+          for (int k = 0; k < C::ATOMS * 4; ++k) {  // +32 bytes per MMA step inside an atom
+            const int a = k / 4, ks = k % 4;
             const uint64_t ao = (uint64_t)((a * (C::A_BYTES / C::ATOMS)) >> 4) + 2 * ks;
             const uint64_t bo = (uint64_t)((a * (C::B_BYTES / C::ATOMS)) >> 4) + 2 * ks;
-            umma_bf16(d_tmem, a0 + ao, b0 + bo, C::IDESC, (kb | k) != 0 ? 1u : 0u);
+            if (F8)
+              umma_e4m3(d_tmem, a0 + ao, b0 + bo, C::IDESC, (kb | k) != 0 ? 1u : 0u);
+            else
+              umma_bf16(d_tmem, a0 + ao, b0 + bo, C::IDESC, (kb | k) != 0 ? 1u : 0u);
           }
           umma_commit(&empty[stage]);
           if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
@@ -454,11 +463,29 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK>::THREADS, 1)
         } else {
           // bias (+ GELU) in the row layout, bf16 to the staging buffer, then
           // whole-row-segment stores
-          float bv[32];
-          if (epi.bias) Vec<bf16, 32>::load(static_cast<const bf16*>(epi.bias) + col, bv);
           float v[32];
+          if (F8) {
+            // E4M3 weights carry one scale per output column: 8 columns at a
+            // time, so that scales and biases do not hold 64 registers
 #pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]) + (epi.bias ? bv[i] : 0.f);
+            for (int g = 0; g < 4; ++g) {
+              float sv[8], bb[8];
+              Vec<float, 8>::load(epi.wscale + col + 8 * g, sv);
+              if (epi.bias) {
+                Vec<bf16, 8>::load(static_cast<const bf16*>(epi.bias) + col + 8 * g, bb);
+              } else {
+#pragma unroll
+                for (int i = 0; i < 8; ++i) bb[i] = 0.f;
+              }
+#pragma unroll
+              for (int i = 0; i < 8; ++i) v[8 * g + i] = fmaf(__uint_as_float(r[8 * g + i]), sv[i], bb[i]);
+            }
+          } else {
+            float bv[32];
+            if (epi.bias) Vec<bf16, 32>::load(static_cast<const bf16*>(epi.bias) + col, bv);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]) + (epi.bias ? bv[i] : 0.f);
+          }
           if (EK == tc::BF16OUT_SILU) {
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = silu(v[i]);
@@ -580,19 +607,22 @@ static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   return fn;
 }
 
-// 2-D bf16 tensor map over a row-major [outer, inner] matrix with the given
-// row pitch, box [box_outer, box_inner], out-of-bounds elements read as zero.
-bool make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t pitch_bytes,
-                    uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swz) {
+// 2-D tensor map over a row-major [outer, inner] matrix with the given row
+// pitch, box [box_outer, box_inner], out-of-bounds elements read as zero.
+static bool make_tmap_2d(CUtensorMapDataType dt, CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
+                         uint64_t pitch_bytes, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swz) {
   auto enc = tensor_map_encoder();
   if (!enc) return false;
   cuuint64_t dims[2] = {inner, outer};
   cuuint64_t strides[1] = {pitch_bytes};
   cuuint32_t box[2] = {box_inner, box_outer};
   cuuint32_t es[2] = {1, 1};
-  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  return enc(m, dt, 2, const_cast<void*>(base), dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+bool make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t pitch_bytes,
+                    uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swz) {
+  return make_tmap_2d(CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, m, base, inner, outer, pitch_bytes, box_inner, box_outer, swz);
 }
 
 bool gemm_supported(int dtype, int M, int N, int K, const GemmEpi& epi, const char** why) {
@@ -602,7 +632,16 @@ bool gemm_supported(int dtype, int M, int N, int K, const GemmEpi& epi, const ch
   if (epi.gate && (epi.mode != LAZYMAR_EPI_RESIDUAL || epi.ldg < N || epi.ldg % 4 != 0)) {
     *why = "a gate needs the residual epilogue and ldg >= N, ldg % 4 == 0"; return false;
   }
-  if (dtype == LAZYMAR_BF16) {
+  if (dtype == LAZYMAR_E4M3) {
+    if (K % 128 != 0) { *why = "E4M3 GEMM needs K % 128 == 0"; return false; }
+    if (N % 128 != 0) { *why = "E4M3 GEMM needs N % 128 == 0"; return false; }
+    if (epi.mode == LAZYMAR_EPI_RESIDUAL || epi.mode == LAZYMAR_EPI_SILU) {
+      *why = "E4M3 GEMM: bias, GELU or Q/K/V epilogue only"; return false;
+    }
+    if (!epi.wscale) { *why = "E4M3 GEMM needs the per-column weight scales"; return false; }
+    if (epi.mode == LAZYMAR_EPI_QKV && epi.D % 32 != 0) { *why = "QKV epilogue needs D % 32 == 0"; return false; }
+    if (epi.mode != LAZYMAR_EPI_QKV && epi.ldo % 8 != 0) { *why = "ldo % 8 == 0 required"; return false; }
+  } else if (dtype == LAZYMAR_BF16) {
     if (K % 64 != 0) { *why = "bf16 GEMM needs K % 64 == 0"; return false; }
     if (N % 128 != 0) { *why = "bf16 GEMM needs N % 128 == 0"; return false; }
     if (epi.mode == LAZYMAR_EPI_QKV && epi.D % 32 != 0) { *why = "QKV epilogue needs D % 32 == 0"; return false; }
@@ -618,20 +657,22 @@ bool gemm_supported(int dtype, int M, int N, int K, const GemmEpi& epi, const ch
   return true;
 }
 
-template <int BN, int EK, int BK>
+template <int BN, int EK, int BK, int F8 = 0>
 static cudaError_t launch_tc(const Ctx& c, const void* A, const void* W, int M, int N, int K, const GemmEpi& epi) {
-  using C = tc::Cfg<BN, EK, BK>;
+  using C = tc::Cfg<BN, EK, BK, F8>;
+  const CUtensorMapDataType dt = F8 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
   CUtensorMap ta, tb;
-  if (!make_tmap_bf16(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * 2, tc::ATOM_K, tc::BM,
-                      CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !make_tmap_bf16(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, tc::ATOM_K, BN, CU_TENSOR_MAP_SWIZZLE_128B))
+  if (!make_tmap_2d(dt, &ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * C::EB, C::ATOM_E, tc::BM,
+                    CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_tmap_2d(dt, &tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * C::EB, C::ATOM_E, BN,
+                    CU_TENSOR_MAP_SWIZZLE_128B))
     return cudaErrorInvalidValue;
   static int attr_set[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc_kernel<BN, EK, BK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)C::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc_kernel<BN, EK, BK, F8>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
     if (e != cudaSuccess) return e;
     attr_set[dev] = 1;
   }
@@ -655,7 +696,7 @@ static cudaError_t launch_tc(const Ctx& c, const void* A, const void* W, int M, 
   }
   const int tiles = ((M + tc::BM - 1) / tc::BM) * (N / BN);
   const int grid = tiles < c.num_sms ? tiles : c.num_sms;
-  return launch_pdl(gemm_bf16_tc_kernel<BN, EK, BK>, dim3(grid), dim3(C::THREADS), C::SMEM, c.stream, ta, tb, to[0], to[1],
+  return launch_pdl(gemm_bf16_tc_kernel<BN, EK, BK, F8>, dim3(grid), dim3(C::THREADS), C::SMEM, c.stream, ta, tb, to[0], to[1],
                     to[2], tma_out, M, N, K,
                     epi, c.err);
 }
@@ -695,6 +736,13 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
         bn = widths[i];
       }
     }
+  }
+  if (dtype == LAZYMAR_E4M3) {
+    // E4M3 operands (bf16-output kinds): a 128-element stage is one atom; the
+    // tile width follows the bf16 choice
+    if (bn == 256) return launch_tc<256, tc::BF16OUT, 128, 1>(c, A, W, M, N, K, epi);
+    if (bn == 192) return launch_tc<192, tc::BF16OUT, 128, 1>(c, A, W, M, N, K, epi);
+    return launch_tc<128, tc::BF16OUT, 128, 1>(c, A, W, M, N, K, epi);
   }
   const int ek = epi.mode == LAZYMAR_EPI_SILU       ? tc::BF16OUT_SILU
                  : epi.mode != LAZYMAR_EPI_RESIDUAL ? tc::BF16OUT

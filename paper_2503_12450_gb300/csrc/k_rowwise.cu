@@ -11,6 +11,8 @@
 //     16-byte vectors.
 // All of these are bound by HBM bandwidth; one warp per row (LayerNorm) or
 // grid-stride 16-byte vectors (CFG) keeps loads coalesced.
+#include <cuda_fp8.h>
+
 #include "lazymar_internal.cuh"
 
 namespace lm {
@@ -182,6 +184,86 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const float* __restrict_
   for (int i = 0; i < NV; ++i) ln_write4<TO>(yr, g, b, 4 * (lane + 32 * i), v[i], mean, rstd);
 }
 
+// Four values to four E4M3 bytes (round to nearest even, saturating at the
+// largest finite value 448), the A operand of an 8-bit GEMM.
+__device__ __forceinline__ uint32_t pack_e4m3x4(float a, float b, float c, float d) {
+  const uint32_t lo = __nv_cvt_float2_to_fp8x2(make_float2(a, b), __NV_SATFINITE, __NV_E4M3);
+  const uint32_t hi = __nv_cvt_float2_to_fp8x2(make_float2(c, d), __NV_SATFINITE, __NV_E4M3);
+  return lo | (hi << 16);
+}
+
+// layernorm_kernel with an E4M3 output (gain and shift in TG): the A operand
+// of the E4M3 Q/K/V projection.
+template <typename TG, int NV>
+__global__ void __launch_bounds__(256) layernorm_e4m3_kernel(const float* __restrict__ x,
+                                                             const int* __restrict__ row_map,
+                                                             const TG* __restrict__ g, const TG* __restrict__ b,
+                                                             uint8_t* __restrict__ y, float* __restrict__ x_copy,
+                                                             int M, int D, float eps) {
+  pdl_wait();
+  pdl_trigger();
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (row >= M) return;
+  const int src = row_map ? row_map[row] : row;
+  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)src * D);
+  float4 v[NV];
+#pragma unroll
+  for (int i = 0; i < NV; ++i) v[i] = xr[lane + 32 * i];
+  if (x_copy) {
+    float4* cr = reinterpret_cast<float4*>(x_copy + (size_t)row * D);
+#pragma unroll
+    for (int i = 0; i < NV; ++i) cr[lane + 32 * i] = v[i];
+  }
+  float mean, rstd;
+  ln_stats<NV>(v, D, eps, mean, rstd);
+  uint8_t* yr = y + (size_t)row * D;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    const int col = 4 * (lane + 32 * i);
+    const float4 gg = load4(g + col), bb = load4(b + col);
+    *reinterpret_cast<uint32_t*>(yr + col) =
+        pack_e4m3x4((v[i].x - mean) * rstd * gg.x + bb.x, (v[i].y - mean) * rstd * gg.y + bb.y,
+                    (v[i].z - mean) * rstd * gg.z + bb.z, (v[i].w - mean) * rstd * gg.w + bb.w);
+  }
+}
+
+// E4M3 weights with one scale per row (output channel): scale = max|w| / 448
+// (1 for an all-zero row), q = e4m3(w / scale). One warp per row.
+__global__ void __launch_bounds__(256) quantize_rows_e4m3_kernel(const bf16* __restrict__ w, int rows, int cols,
+                                                                 uint8_t* __restrict__ q, float* __restrict__ scale) {
+  pdl_wait();
+  pdl_trigger();
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const bf16* wr = w + (size_t)row * cols;
+  float amax = 0.f;
+  for (int k = lane * 8; k < cols; k += 256) {
+    float f[8];
+    Vec<bf16, 8>::load(wr + k, f);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) amax = fmaxf(amax, fabsf(f[i]));
+  }
+  amax = warp_max(amax);
+  const float s = amax > 0.f ? amax / 448.f : 1.f;
+  if (lane == 0) scale[row] = s;
+  uint8_t* qr = q + (size_t)row * cols;
+  for (int k = lane * 8; k < cols; k += 256) {
+    float f[8];
+    Vec<bf16, 8>::load(wr + k, f);
+    uint2 u;
+    u.x = pack_e4m3x4(f[0] / s, f[1] / s, f[2] / s, f[3] / s);
+    u.y = pack_e4m3x4(f[4] / s, f[5] / s, f[6] / s, f[7] / s);
+    *reinterpret_cast<uint2*>(qr + k) = u;
+  }
+}
+
+cudaError_t launch_quantize_e4m3(const Ctx& c, const void* w, int rows, int cols, void* q, float* scale) {
+  if (rows == 0) return cudaSuccess;
+  if (cols % 8 != 0) return cudaErrorInvalidValue;
+  return launch_pdl(quantize_rows_e4m3_kernel, dim3((unsigned)((rows + 7) / 8)), dim3(256), 0, c.stream,
+                    static_cast<const bf16*>(w), rows, cols, static_cast<uint8_t*>(q), scale);
+}
+
 template <typename TO, int NV>
 __global__ void __launch_bounds__(256) final_ln_kernel(const float* __restrict__ x, const int* __restrict__ row_map,
                                                        int T, int nb, int n_img, const TO* __restrict__ g,
@@ -227,7 +309,11 @@ cudaError_t launch_layernorm(const Ctx& c, int dtype, const float* x, const int*
                              const void* b, void* y, float* x_copy, int M, int D, float eps) {
   if (M == 0) return cudaSuccess;
   const unsigned grid = (unsigned)((M + 7) / 8);
-  if (dtype == LAZYMAR_BF16) {
+  if (dtype == LAZYMAR_E4M3) {
+    // bf16 gain and shift, E4M3 output
+    LM_LN_DISPATCH(layernorm_e4m3_kernel, bf16, x, row_map, (const bf16*)g, (const bf16*)b, (uint8_t*)y, x_copy, M,
+                   D, eps)
+  } else if (dtype == LAZYMAR_BF16) {
     LM_LN_DISPATCH(layernorm_kernel, bf16, x, row_map, (const bf16*)g, (const bf16*)b, (bf16*)y, x_copy, M, D, eps)
   } else {
     LM_LN_DISPATCH(layernorm_kernel, float, x, row_map, (const float*)g, (const float*)b, (float*)y, x_copy, M, D,

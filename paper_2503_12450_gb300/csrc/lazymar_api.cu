@@ -104,6 +104,11 @@ struct lazymar_handle {
   // token cache: keys/values of blocks s..L-1; selection reference; output
   // features of the image tokens; condition cache
   std::vector<void*> Kc, Vc;
+  // qkv_e4m3: E4M3 copies of W_qkv of blocks s..L-1 with per-row scales, and
+  // the E4M3 LN1 output of the recomputed tokens
+  std::vector<uint8_t*> wq8;
+  std::vector<float*> wsc;
+  uint8_t* A8 = nullptr;
   void *ref = nullptr, *zc = nullptr, *delta = nullptr;
   // scratch
   float *H = nullptr, *Hc = nullptr;
@@ -253,6 +258,9 @@ lazymar_status check_config(const lazymar_config* c) {
   if (c->sel_layers < 1 || c->sel_layers > c->depth)
     return fail(LAZYMAR_ERR_INVALID_ARG, "config: 1 <= sel_layers <= depth required");
   if (c->token_dim < 1 || c->token_dim > 64) return fail(LAZYMAR_ERR_UNSUPPORTED, "config: token_dim must be 1..64");
+  if (c->qkv_e4m3 != 0 && c->qkv_e4m3 != 1) return fail(LAZYMAR_ERR_INVALID_ARG, "config: qkv_e4m3 must be 0 or 1");
+  if (c->qkv_e4m3 && (c->dtype != LAZYMAR_BF16 || c->width % 128 != 0))
+    return fail(LAZYMAR_ERR_UNSUPPORTED, "config: qkv_e4m3 needs bf16 and width % 128 == 0");
   if (c->width % c->heads != 0) return fail(LAZYMAR_ERR_INVALID_ARG, "config: heads must divide width");
   if (!layernorm_width_ok(c->width))
     return fail(LAZYMAR_ERR_UNSUPPORTED, "config: width must be 128 * {1,2,4,6,8,10,12,16}");
@@ -306,6 +314,15 @@ extern "C" lazymar_status lazymar_create(const lazymar_config* cfg, const lazyma
     o_k[l] = b.take(rowsT * D * es);
     o_v[l] = b.take(rowsT * D * es);
   }
+  std::vector<size_t> o_wq8(h->L, 0), o_wsc(h->L, 0);
+  size_t o_A8 = 0;
+  if (cfg->qkv_e4m3) {
+    for (int l = h->s; l < h->L; ++l) {
+      o_wq8[l] = b.take(3 * D * D);
+      o_wsc[l] = b.take(3 * D * 4);
+    }
+    o_A8 = b.take(rowsT * D);
+  }
   const size_t o_ref = b.take(rowsT * D * es), o_zc = b.take(R * cfg->n_img * D * es),
                o_delta = b.take(Bm * cfg->n_img * D * es);
   // scratch
@@ -348,6 +365,15 @@ extern "C" lazymar_status lazymar_create(const lazymar_config* cfg, const lazyma
     h->Vc[l] = a + o_v[l];
   }
   h->ref = a + o_ref; h->zc = a + o_zc; h->delta = a + o_delta;
+  h->wq8.assign(h->L, nullptr);
+  h->wsc.assign(h->L, nullptr);
+  if (cfg->qkv_e4m3) {
+    for (int l = h->s; l < h->L; ++l) {
+      h->wq8[l] = a + o_wq8[l];
+      h->wsc[l] = reinterpret_cast<float*>(a + o_wsc[l]);
+    }
+    h->A8 = a + o_A8;
+  }
   h->H = reinterpret_cast<float*>(a + o_H); h->Hc = reinterpret_cast<float*>(a + o_Hc);
   h->A = a + o_A; h->Q = a + o_Q; h->Ks = a + o_Ks; h->Vs = a + o_Vs; h->O = a + o_O; h->U = a + o_U;
   h->Fs = a + o_Fs;
@@ -383,6 +409,15 @@ extern "C" lazymar_status lazymar_create(const lazymar_config* cfg, const lazyma
         (st = upload(bd.w1, s.w1, H4 * D, dt)) || (st = upload(bd.b1, s.b1, H4, dt)) ||
         (st = upload(bd.w2, s.w2, D * H4, dt)) || (st = upload(bd.b2, s.b2, D, dt)))
       return destroy(st);
+  }
+  if (cfg->qkv_e4m3) {
+    const Ctx qc{h->gstream, h->err, h->num_sms};
+    for (int l = h->s; l < h->L; ++l) {
+      e = launch_quantize_e4m3(qc, h->blk[l].w_qkv, 3 * (int)D, (int)D, h->wq8[l], h->wsc[l]);
+      if (e != cudaSuccess) return destroy(cuda_fail(e, "E4M3 weight quantization"));
+    }
+    e = cudaStreamSynchronize(h->gstream);
+    if (e != cudaSuccess) return destroy(cuda_fail(e, "E4M3 weight quantization"));
   }
   *out = h;
   return LAZYMAR_OK;
@@ -442,18 +477,22 @@ double gemm_bytes(const lazymar_handle* h, int M, int N, int K, int mode) {
 }
 
 lazymar_status gemm(lazymar_handle* h, const Ctx& c, const void* A, const void* W, int M, int N, int K,
-                    const GemmEpi& e) {
+                    const GemmEpi& e, int dtype = -1) {
   if (M == 0) return LAZYMAR_OK;
-  return launch(h, LAZYMAR_K_GEMM, 2.0 * M * N * K, gemm_bytes(h, M, N, K, e.mode), c.stream, "gemm",
-                [&] { return launch_gemm(c, h->cfg.dtype, A, W, M, N, K, e, 0); });
+  const int dt = dtype < 0 ? h->cfg.dtype : dtype;
+  double bytes = gemm_bytes(h, M, N, K, e.mode);
+  if (dt == LAZYMAR_E4M3) bytes -= (double)h->es * ((double)M * K + (double)N * K) / 2.0;  // 1-byte operands
+  return launch(h, LAZYMAR_K_GEMM, 2.0 * M * N * K, bytes, c.stream, "gemm",
+                [&] { return launch_gemm(c, dt, A, W, M, N, K, e, 0); });
 }
 
 lazymar_status layernorm(lazymar_handle* h, const Ctx& c, const float* x, const int* map, const void* g, const void* b,
-                         void* y, float* copy, int M) {
+                         void* y, float* copy, int M, int dtype = -1) {
   if (M == 0) return LAZYMAR_OK;
-  const double bytes = (double)M * h->D * (4.0 + h->es + (copy ? 4.0 : 0.0));
+  const int dt = dtype < 0 ? h->cfg.dtype : dtype;
+  const double bytes = (double)M * h->D * (4.0 + (dt == LAZYMAR_E4M3 ? 1.0 : h->es) + (copy ? 4.0 : 0.0));
   return launch(h, LAZYMAR_K_LAYERNORM, 0, bytes, c.stream, "layernorm", [&] {
-    return launch_layernorm(c, h->cfg.dtype, x, map, g, b, y, copy, M, h->D, h->cfg.ln_eps);
+    return launch_layernorm(c, dt, x, map, g, b, y, copy, M, h->D, h->cfg.ln_eps);
   });
 }
 
@@ -487,12 +526,24 @@ lazymar_status layer_full(lazymar_handle* h, const Ctx& c, int l, int rows, void
 lazymar_status layer_cached(lazymar_handle* h, const Ctx& c, int l, int rows, int N, bool first) {
   const BlockDev& b = h->blk[l];
   const int M = rows * N, D = h->D;
-  if (first)
-    LM_TRY(layernorm(h, c, h->H, h->row_map, b.ln1_g, b.ln1_b, h->A, h->Hc, M));
-  else
-    LM_TRY(layernorm(h, c, h->Hc, nullptr, b.ln1_g, b.ln1_b, h->A, nullptr, M));
-  LM_TRY(gemm(h, c, h->A, b.w_qkv, M, 3 * D, D,
-              GemmEpi{LAZYMAR_EPI_QKV, b.b_qkv, h->Q, D, h->Kc[l], h->Vc[l], h->row_map, D}));
+  if (h->cfg.qkv_e4m3) {
+    // LN1 to E4M3, then the 8-bit Q/K/V projection with per-channel scales
+    const int e8 = LAZYMAR_E4M3;
+    if (first)
+      LM_TRY(layernorm(h, c, h->H, h->row_map, b.ln1_g, b.ln1_b, h->A8, h->Hc, M, e8));
+    else
+      LM_TRY(layernorm(h, c, h->Hc, nullptr, b.ln1_g, b.ln1_b, h->A8, nullptr, M, e8));
+    GemmEpi qe{LAZYMAR_EPI_QKV, b.b_qkv, h->Q, D, h->Kc[l], h->Vc[l], h->row_map, D};
+    qe.wscale = h->wsc[l];
+    LM_TRY(gemm(h, c, h->A8, h->wq8[l], M, 3 * D, D, qe, e8));
+  } else {
+    if (first)
+      LM_TRY(layernorm(h, c, h->H, h->row_map, b.ln1_g, b.ln1_b, h->A, h->Hc, M));
+    else
+      LM_TRY(layernorm(h, c, h->Hc, nullptr, b.ln1_g, b.ln1_b, h->A, nullptr, M));
+    LM_TRY(gemm(h, c, h->A, b.w_qkv, M, 3 * D, D,
+                GemmEpi{LAZYMAR_EPI_QKV, b.b_qkv, h->Q, D, h->Kc[l], h->Vc[l], h->row_map, D}));
+  }
   LM_TRY(attention(h, c, h->Kc[l], h->Vc[l], rows, N));
   LM_TRY(gemm(h, c, h->O, b.w_o, M, D, D, GemmEpi{LAZYMAR_EPI_RESIDUAL, b.b_o, h->Hc, D, nullptr, nullptr, nullptr, D}));
   LM_TRY(layernorm(h, c, h->Hc, nullptr, b.ln2_g, b.ln2_b, h->A, nullptr, M));
@@ -814,6 +865,46 @@ extern "C" lazymar_status lazymar_linear(int dtype, int epilogue, const void* a,
   return err == cudaSuccess ? LAZYMAR_OK : cuda_fail(err, "gemm kernel");
 }
 
+extern "C" lazymar_status lazymar_linear_e4m3(int epilogue, const void* a, const void* w, const float* wscale,
+                                              const void* bias, int M, int N, int K, void* out, int ldo, void* k_out,
+                                              void* v_out, const int32_t* row_map, int flags, void* stream) {
+  if (epilogue != LAZYMAR_EPI_BIAS && epilogue != LAZYMAR_EPI_GELU && epilogue != LAZYMAR_EPI_QKV)
+    return fail(LAZYMAR_ERR_INVALID_ARG, "epilogue: BIAS, GELU or QKV");
+  if (flags < 0 || flags > 4) return fail(LAZYMAR_ERR_INVALID_ARG, "flags");
+  GemmEpi e{epilogue, bias, out, ldo, k_out, v_out, row_map, epilogue == LAZYMAR_EPI_QKV ? N / 3 : 0};
+  e.wscale = wscale;
+  const char* why = "";
+  if (!gemm_supported(LAZYMAR_E4M3, M, N, K, e, &why)) return fail(LAZYMAR_ERR_UNSUPPORTED, why);
+  if (epilogue != LAZYMAR_EPI_QKV && ldo < N) return fail(LAZYMAR_ERR_INVALID_ARG, "ldo < N");
+  if (M == 0) return LAZYMAR_OK;
+  if (!is_device_ptr(a) || !is_device_ptr(w) || !is_device_ptr(wscale) || !is_device_ptr(out) ||
+      (bias && !is_device_ptr(bias)))
+    return fail(LAZYMAR_ERR_INVALID_ARG, "a, w, wscale, bias and out must be device pointers");
+  if (epilogue == LAZYMAR_EPI_QKV && (!is_device_ptr(k_out) || !is_device_ptr(v_out)))
+    return fail(LAZYMAR_ERR_INVALID_ARG, "k_out and v_out must be device pointers");
+  const void* ps[] = {a, w, wscale, bias, out, k_out, v_out};
+  for (const void* p : ps)
+    if (p && !aligned16(p)) return fail(LAZYMAR_ERR_INVALID_ARG, "16-byte alignment required");
+  Ctx c;
+  LM_TRY(component_ctx(stream, &c));
+  cudaError_t err = launch_gemm(c, LAZYMAR_E4M3, a, w, M, N, K, e, flags);
+  return err == cudaSuccess ? LAZYMAR_OK : cuda_fail(err, "E4M3 gemm kernel");
+}
+
+extern "C" lazymar_status lazymar_quantize_e4m3(const void* w, int rows, int cols, void* q, float* scale,
+                                                void* stream) {
+  if (rows < 0 || cols < 8 || cols % 8 != 0) return fail(LAZYMAR_ERR_INVALID_ARG, "rows >= 0, cols % 8 == 0 required");
+  if (rows == 0) return LAZYMAR_OK;
+  if (!is_device_ptr(w) || !is_device_ptr(q) || !is_device_ptr(scale))
+    return fail(LAZYMAR_ERR_INVALID_ARG, "device pointers required");
+  if (!aligned16(w) || (reinterpret_cast<uintptr_t>(q) & 7u))
+    return fail(LAZYMAR_ERR_INVALID_ARG, "w 16-byte and q 8-byte alignment required");
+  Ctx c;
+  LM_TRY(component_ctx(stream, &c));
+  cudaError_t e = launch_quantize_e4m3(c, w, rows, cols, q, scale);
+  return e == cudaSuccess ? LAZYMAR_OK : cuda_fail(e, "E4M3 quantization kernel");
+}
+
 extern "C" lazymar_status lazymar_attention(int dtype, const void* q, const void* k, const void* v, void* o, int rows,
                                             int n_q, int T, int heads, int head_dim, void* stream) {
   const char* why = "";
@@ -834,7 +925,8 @@ extern "C" lazymar_status lazymar_attention(int dtype, const void* q, const void
 
 extern "C" lazymar_status lazymar_layernorm(int dtype, const float* x, const int32_t* row_map, const void* g,
                                             const void* b, void* y, int M, int D, float eps, void* stream) {
-  if (dtype != LAZYMAR_F32 && dtype != LAZYMAR_BF16) return fail(LAZYMAR_ERR_INVALID_ARG, "dtype");
+  if (dtype != LAZYMAR_F32 && dtype != LAZYMAR_BF16 && dtype != LAZYMAR_E4M3)
+    return fail(LAZYMAR_ERR_INVALID_ARG, "dtype");
   if (M < 0 || !layernorm_width_ok(D) || !(eps > 0.f))
     return fail(LAZYMAR_ERR_UNSUPPORTED, "M >= 0, D = 128 * {1,2,4,6,8,10,12,16}, eps > 0 required");
   if (M == 0) return LAZYMAR_OK;

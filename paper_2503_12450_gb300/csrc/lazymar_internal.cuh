@@ -325,6 +325,16 @@ __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint6
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// D[tmem] (+)= A[smem] * B[smem]^T, E4M3 inputs, fp32 accumulate (kind::f8f6f4).
+__device__ __forceinline__ void umma_e4m3(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
 // Arrive on `bar` once all tcgen05.mma previously issued by this thread complete.
 __device__ __forceinline__ void umma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
@@ -427,6 +437,9 @@ struct GemmEpi {
   // gated residual of an adaptive-LayerNorm block), or nullptr for out += y
   const void* gate;
   int ldg;
+  // E4M3 operands only: per-column scale of the weights ([N] fp32), applied
+  // to the accumulator before the bias
+  const float* wscale;
 };
 cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, int M, int N, int K,
                         const GemmEpi& epi, int flags);
@@ -437,6 +450,8 @@ cudaError_t launch_attention(const Ctx& c, int dtype, const void* q, const void*
                              int rows, int n_q, int T, int heads, int dh);
 bool attention_supported(int dtype, int heads, int dh, const char** why);
 
+// dtype LAZYMAR_E4M3: bf16 gain/shift, E4M3 output (the A operand of an
+// 8-bit GEMM); otherwise gain, shift and output in dtype.
 cudaError_t launch_layernorm(const Ctx& c, int dtype, const float* x, const int* row_map, const void* g,
                              const void* b, void* y, float* x_copy, int M, int D, float eps);
 // Final LayerNorm of compact rows into the [rows, n_img, D] output cache:
@@ -449,6 +464,9 @@ cudaError_t launch_embed(const Ctx& c, int dtype, const float* lat, const uint8_
                          float* H, int rows, int B, int T, int n_buffer, int n_img, int D, int token_dim,
                          int n_classes);
 cudaError_t launch_cast(const Ctx& c, int dtype, const float* x, void* y, size_t n);
+// E4M3 copy of a bf16 weight matrix [rows, cols] with one scale per row
+// (max |w| / 448): q [rows, cols] bytes, scale [rows] fp32.
+cudaError_t launch_quantize_e4m3(const Ctx& c, const void* w, int rows, int cols, void* q, float* scale);
 
 cudaError_t launch_similarity(const Ctx& c, int dtype, const void* cur, void* cache, double* S, int rows, int T,
                               int D, bool copy);

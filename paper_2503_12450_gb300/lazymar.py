@@ -12,7 +12,7 @@ import os
 HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "liblazymar.so")
 
-LAZYMAR_F32, LAZYMAR_BF16 = 0, 1
+LAZYMAR_F32, LAZYMAR_BF16, LAZYMAR_E4M3 = 0, 1, 2
 LAZYMAR_CRITERION_VALUE, LAZYMAR_CRITERION_FEATURE = 0, 1
 LAZYMAR_SELECT_LEAST_SIMILAR, LAZYMAR_SELECT_MOST_SIMILAR, LAZYMAR_SELECT_RANDOM = 0, 1, 2
 LAZYMAR_CFG_GUIDE, LAZYMAR_CFG_REFRESH, LAZYMAR_CFG_REUSE = 0, 1, 2
@@ -31,7 +31,7 @@ class LazymarError(RuntimeError):
 class lazymar_config(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int) for n in ("depth", "width", "heads", "mlp_ratio", "n_buffer", "n_img", "token_dim",
                                              "n_classes", "max_batch", "sel_layers", "dtype", "criterion")] + [
-        ("ln_eps", ctypes.c_float), ("select_rule", ctypes.c_int)]
+        ("ln_eps", ctypes.c_float), ("select_rule", ctypes.c_int), ("qkv_e4m3", ctypes.c_int)]
 
 
 _FP = ctypes.c_void_p
@@ -106,6 +106,8 @@ def lib():
         "lazymar_cfg_combine": (st, [i, i, vp, vp, vp, f, sz, vp, vp, vp]),
         "lazymar_linear": (st, [i, i, vp, vp, vp, i, i, i, vp, i, vp, vp, vp, i, vp]),
         "lazymar_attention": (st, [i, vp, vp, vp, vp, i, i, i, i, i, vp]),
+        "lazymar_linear_e4m3": (st, [i, vp, vp, vp, vp, i, i, i, vp, i, vp, vp, vp, i, vp]),
+        "lazymar_quantize_e4m3": (st, [vp, i, i, vp, vp, vp]),
         "lazymar_layernorm": (st, [i, vp, vp, vp, vp, vp, i, i, f, vp]),
         "lazymar_plan_step": (i, [i, i, i, i, i]),
         "lazymar_sync": (st, [vp, vp]),
@@ -174,7 +176,7 @@ def lazymar_create(cfg, weights):
     arrays or torch tensors as produced by synth.make_weights. Returns a Handle."""
     c = lazymar_config()
     for n, _ in lazymar_config._fields_:
-        if n in ("dtype", "criterion", "ln_eps", "select_rule"):
+        if n in ("dtype", "criterion", "ln_eps", "select_rule", "qkv_e4m3"):
             continue
         setattr(c, n, int(cfg[n] if n != "max_batch" else cfg.get("max_batch", cfg.get("batch"))))
     dt = cfg["dtype"]
@@ -185,6 +187,7 @@ def lazymar_create(cfg, weights):
     sr = cfg.get("select_rule", LAZYMAR_SELECT_LEAST_SIMILAR)
     c.select_rule = {"least_similar": LAZYMAR_SELECT_LEAST_SIMILAR, "most_similar": LAZYMAR_SELECT_MOST_SIMILAR,
                      "random": LAZYMAR_SELECT_RANDOM}.get(sr, sr)
+    c.qkv_e4m3 = int(bool(cfg.get("qkv_e4m3", 0)))
     keep = []
 
     def p(a):
@@ -256,6 +259,17 @@ def lazymar_linear(dtype, epilogue, a, w, bias, M, N, K, out, ldo, k_out=None, v
     _check(lib().lazymar_linear(int(dtype), int(epilogue), _ptr(a), _ptr(w), _ptr(bias), int(M), int(N), int(K),
                                 _ptr(out), int(ldo), _ptr(k_out), _ptr(v_out), _ptr(row_map), int(flags),
                                 _stream(stream)))
+
+
+def lazymar_linear_e4m3(epilogue, a, w, wscale, bias, M, N, K, out, ldo, k_out=None, v_out=None, row_map=None,
+                        flags=0, stream=None):
+    _check(lib().lazymar_linear_e4m3(int(epilogue), _ptr(a), _ptr(w), _ptr(wscale), _ptr(bias), int(M), int(N),
+                                     int(K), _ptr(out), int(ldo), _ptr(k_out), _ptr(v_out), _ptr(row_map), int(flags),
+                                     _stream(stream)))
+
+
+def lazymar_quantize_e4m3(w, rows, cols, q, scale, stream=None):
+    _check(lib().lazymar_quantize_e4m3(_ptr(w), int(rows), int(cols), _ptr(q), _ptr(scale), _stream(stream)))
 
 
 def lazymar_attention(dtype, q, k, v, o, rows, n_q, T, heads, head_dim, stream=None):

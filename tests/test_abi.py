@@ -66,7 +66,8 @@ def _cfg(**kw):
 @pytest.mark.parametrize("bad,status", [(dict(sel_layers=0), 1), (dict(sel_layers=3), 1), (dict(width=200), 6),
                                         (dict(width=384, heads=3), 6), (dict(heads=2, dtype="bf16"), 6),
                                         (dict(token_dim=65), 6), (dict(max_batch=0), 1), (dict(dtype=7), 1),
-                                        (dict(select_rule=3), 1)])
+                                        (dict(select_rule=3), 1), (dict(qkv_e4m3=2), 1),
+                                        (dict(qkv_e4m3=1), 6)])
 def test_create_rejects_bad_configs_before_touching_the_device(lib, bad, status):
     with pytest.raises(lm.LazymarError) as e:
         _create_raw(lib, _cfg(**bad))
@@ -76,8 +77,9 @@ def test_create_rejects_bad_configs_before_touching_the_device(lib, bad, status)
 def _create_raw(lib, cfg):
     c = lm.lazymar_config()
     for n, _ in lm.lazymar_config._fields_:
-        if n not in ("dtype", "criterion", "ln_eps", "select_rule"):
+        if n not in ("dtype", "criterion", "ln_eps", "select_rule", "qkv_e4m3"):
             setattr(c, n, cfg[n])
+    c.qkv_e4m3 = cfg.get("qkv_e4m3", 0)
     c.dtype = {"fp32": 0, "bf16": 1}.get(cfg["dtype"], cfg["dtype"])
     c.criterion = 0
     c.ln_eps = 1e-6

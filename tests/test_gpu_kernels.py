@@ -5,6 +5,7 @@ import pytest
 
 import oracle as O
 from oracle import diffusion_head as HO
+from oracle import fp8
 import synth
 from paper_2503_12450_gb300 import lazymar as lm
 from _gpu import DT, TOL, dev, dev_int, empty, host, max_rel, sync, torch_cuda
@@ -260,6 +261,111 @@ def test_linear_fp32(M, N, K, epi):
     if epi == lm.LAZYMAR_EPI_QKV and (N % 3 or (N // 3) % 4):
         pytest.skip("not a QKV shape")
     _linear_case("fp32", epi, M, N, K, 0, seed=M + N + K + epi)
+
+
+# --------------------------------------------------------------------------
+# E4M3 Q/K/V projection (qkv_e4m3): weight quantization, LayerNorm to E4M3,
+# the kind::f8f6f4 GEMM
+# --------------------------------------------------------------------------
+
+def _e4m3_codes(shape, seed):
+    """Random E4M3 bytes over the whole finite range (no NaN codes)."""
+    c = np.random.default_rng(seed).integers(0, 256, size=shape).astype(np.uint8)
+    c[(c & 0x7F) == 0x7F] = 0x38
+    return c
+
+
+@pytest.mark.parametrize("rows,cols", [(2304, 768), (3840, 1280), (5, 8), (130, 1024)])
+def test_quantize_e4m3_bit_exact(rows, cols):
+    """Per-row scales and E4M3 codes of a bf16 weight matrix. The rounding
+    decision is taken in fp32 on both sides (the kernel's precision): scale =
+    fp32(max|w|) / 448, code = E4M3(fp32(w) / scale); the oracle's rounding is
+    the format's definition. Rows of zeros, a row with an exact tie and
+    mixed magnitudes included."""
+    torch = torch_cuda()
+    w = synth.tensor((rows, cols), rows + cols, std=0.02, dtype="bf16")
+    w[0] = 0.0
+    if rows > 2:
+        w[1] = synth.round_bf16(np.linspace(-3, 3, cols).astype(np.float32))
+        w[2] = synth.round_bf16(w[2] * np.float32(1e4))
+    gw = dev(w, "bf16")
+    q = torch.zeros((rows, cols), dtype=torch.uint8, device="cuda")
+    sc = torch.zeros(rows, dtype=torch.float32, device="cuda")
+    lm.lazymar_quantize_e4m3(gw, rows, cols, q, sc)
+    sync()
+    amax = np.abs(w).max(axis=1).astype(np.float32)
+    s32 = np.where(amax > 0, amax / np.float32(448.0), np.float32(1.0)).astype(np.float32)
+    np.testing.assert_array_equal(sc.cpu().numpy(), s32)
+    expect = fp8.e4m3_round((w.astype(np.float32) / s32[:, None]).astype(np.float32))
+    got = fp8.e4m3_decode(q.cpu().numpy())
+    np.testing.assert_array_equal(np.abs(got), np.abs(expect))
+    nz = expect != 0
+    assert (np.sign(got[nz]) == np.sign(expect[nz])).all()
+
+
+def test_layernorm_e4m3_output():
+    """LayerNorm rows to E4M3 (unit scale): every code is the E4M3 rounding of
+    the oracle's LayerNorm, or its neighbour where the fp32 value lies within
+    rounding distance of the midpoint between two codes."""
+    torch = torch_cuda()
+    M, D = 300, 768
+    x = synth.tensor((M, D), 41, std=3.0, mean=0.5)
+    g = synth.tensor((D,), 42, std=0.5, mean=1.0, dtype="bf16")
+    b = synth.tensor((D,), 43, std=0.2, dtype="bf16")
+    y = torch.zeros((M, D), dtype=torch.uint8, device="cuda")
+    lm.lazymar_layernorm(lm.LAZYMAR_E4M3, dev(x), None, dev(g, "bf16"), dev(b, "bf16"), y, M, D, 1e-6)
+    sync()
+    ref = O.layer_norm(x, g, b, 1e-6)
+    got = fp8.e4m3_decode(y.cpu().numpy())
+    exact = fp8.e4m3_round(ref)
+    bad = got != exact
+    assert bad.mean() < 1e-3
+    # where they differ, the oracle's value sits at a rounding midpoint of the two codes
+    lo, hi = np.minimum(got[bad], exact[bad]), np.maximum(got[bad], exact[bad])
+    mid = (lo + hi) / 2
+    assert (np.abs(ref[bad] - mid) <= 1e-5 * np.maximum(np.abs(mid), 1.0)).all()
+    assert (hi - lo <= np.maximum(np.abs(hi), np.abs(lo)) * 2.0 ** -3 + 2.0 ** -9).all()
+
+
+@pytest.mark.parametrize("M,N,K", [(3200, 2304, 768), (1600, 2304, 768), (12800, 3840, 1280), (777, 3072, 1024),
+                                   (1, 384, 128), (130, 256, 256)])
+@pytest.mark.parametrize("epi", [lm.LAZYMAR_EPI_BIAS, lm.LAZYMAR_EPI_QKV])
+def test_linear_e4m3(M, N, K, epi):
+    """The kind::f8f6f4 GEMM on E4M3 operands with per-column weight scales
+    against the oracle's product of the decoded operands (exact in fp64; the
+    GPU accumulates in fp32 and writes bf16), every tile width."""
+    if epi == lm.LAZYMAR_EPI_QKV and (N % 3 or (N // 3) % 32):
+        pytest.skip("not a QKV shape")
+    torch = torch_cuda()
+    seed = M + N + K + epi
+    ac, wc = _e4m3_codes((M, K), seed), _e4m3_codes((N, K), seed + 1)   # subnormals to +-448
+    scale = (np.random.default_rng(seed + 2).uniform(0.5, 2.0, N) * 1e-3).astype(np.float32)
+    bias = synth.tensor((N,), seed + 3, std=0.1, dtype="bf16")
+    ref = fp8.e4m3_decode(ac) @ (fp8.e4m3_decode(wc) * scale[:, None].astype(np.float64)).T + bias
+    ga = torch.from_numpy(ac).cuda()
+    gw = torch.from_numpy(wc).cuda()
+    gs = torch.from_numpy(scale).cuda()
+    gb = dev(bias, "bf16")
+    for flags in [1] + ([2] if N % 256 == 0 else []) + ([3] if N % 192 == 0 else []):
+        if epi == lm.LAZYMAR_EPI_BIAS:
+            out = empty((M, N), "bf16")
+            lm.lazymar_linear_e4m3(epi, ga, gw, gs, gb, M, N, K, out, N, flags=flags)
+            sync()
+            assert max_rel(host(out), ref) < 1e-2, flags
+        else:
+            D = N // 3
+            R = M + 17
+            row_map = synth.distinct_rows(M, R, seed + 4)
+            k0 = synth.tensor((R, D), seed + 5, dtype="bf16")
+            v0 = synth.tensor((R, D), seed + 6, dtype="bf16")
+            q, gk, gv = empty((M, D), "bf16"), dev(k0, "bf16"), dev(v0, "bf16")
+            lm.lazymar_linear_e4m3(epi, ga, gw, gs, gb, M, N, K, q, D, gk, gv, dev_int(row_map), flags=flags)
+            sync()
+            assert max_rel(host(q), ref[:, :D]) < 1e-2
+            k, v = host(gk), host(gv)
+            assert max_rel(k[row_map], ref[:, D:2 * D]) < 1e-2 and max_rel(v[row_map], ref[:, 2 * D:]) < 1e-2
+            keep = np.setdiff1d(np.arange(R), row_map)
+            assert np.array_equal(k[keep], k0[keep]) and np.array_equal(v[keep], v0[keep])
 
 
 # --------------------------------------------------------------------------

@@ -302,8 +302,8 @@ def check_selection(gpu_rows, S_ref, N):
     return overlaps
 
 
-def run_bf16(name, pairs, reuse, n_before=100, n_after=104):
-    r = Run(name)
+def run_bf16(name, pairs, reuse, n_before=100, n_after=104, **over):
+    r = Run(name, **over)
     cfg, B = r.cfg, r.B
     n_img = cfg["n_img"]
     n_before = min(n_before, n_img - 8)
@@ -492,6 +492,17 @@ def test_profiling_times_every_launch_and_changes_no_result():
         assert st[name]["launches"] > 0 and st[name]["timed_launches"] == st[name]["launches"], name
         assert st[name]["ms"] > 0, name
     r.h.close()
+
+
+@pytest.mark.parametrize("name,pairs,reuse,n_before", [("mar_b", [0, 31], True, 100), ("mar_l", [5], True, 100),
+                                                        ("mar_h", [0], True, 100), ("hires", [3], False, 400)])
+def test_steps_with_e4m3_qkv(name, pairs, reuse, n_before):
+    """The same step parity as above with the Q/K/V projection of the cached
+    blocks on 8-bit tensor cores (qkv_e4m3): LN1 output and weights rounded
+    to E4M3. The oracle is the fp64 method; the bf16 tolerance must still
+    hold."""
+    rep = run_bf16(name, pairs=pairs, reuse=reuse, n_before=n_before, qkv_e4m3=1)
+    print(name, "with E4M3 Q/K/V: selection overlap with the oracle:", rep)
 
 
 def test_graph_replay_matches_eager_execution():
