@@ -336,22 +336,29 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
       const int c0 = half * CHUNKS;
       // residual of a 32-column chunk in the coalesced layout: [16-col half][pass]
       float4 res[2][4];
+      uint2 rbias[2];  // the 4 bias values of this lane's columns in each 16-column half (bf16)
       auto load_res = [&](int col) {
 #pragma unroll
-        for (int h = 0; h < 2; ++h)
+        for (int h = 0; h < 2; ++h) {
+          rbias[h] = epi.bias ? *reinterpret_cast<const uint2*>(static_cast<const bf16*>(epi.bias) + col + h * 16 + cq * 4)
+                              : make_uint2(0u, 0u);
 #pragma unroll
           for (int p = 0; p < 4; ++p) {
             const int row = rbase + p * 8 + cr;
             res[h][p] = row < M ? *reinterpret_cast<const float4*>(res_base + (size_t)row * epi.ldo + col + h * 16 + cq * 4)
                                 : make_float4(0.f, 0.f, 0.f, 0.f);
           }
+        }
       };
       // RESID_WIDE layout: [pass] with 4 rows x 8 blocks of 16 bytes per pass
       // (gated kind: the gates of the same elements, prefetched alike)
       float4 resw[8];
       uint2 gatew[8];  // 4 bf16 gates each
+      uint2 wbias;     // the 4 bias values of this lane's columns (bf16)
       auto load_resw = [&](int col) {
         const int wr = lane >> 3, wq = lane & 7;
+        wbias = epi.bias ? *reinterpret_cast<const uint2*>(static_cast<const bf16*>(epi.bias) + col + wq * 4)
+                         : make_uint2(0u, 0u);
 #pragma unroll
         for (int p = 0; p < 8; ++p) {
           const int row = rbase + p * 4 + wr;
@@ -363,8 +370,20 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
                                : make_uint2(0u, 0u);
         }
       };
+      // bf16-output kinds: the bias of the next 32-column chunk (packed bf16),
+      // loaded before it is needed, the first chunk's before the accumulator
+      // is ready
+      uint4 bpre[4];
+      auto load_bias = [&](int col) {
+        if (epi.bias) {
+          const uint4* bp = reinterpret_cast<const uint4*>(static_cast<const bf16*>(epi.bias) + col);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) bpre[j] = bp[j];
+        }
+      };
       if (EK == tc::RESID_HALF) load_res(n0 + c0 * 32);
       if (tc::is_wide<EK>()) load_resw(n0 + c0 * 32);
+      if (tc::is_bf16out<EK>() && !F8) load_bias(n0 + c0 * 32);
       const bool ok = mbar_wait(&acc_full[buf], use, abort_flag, err);
       if (__any_sync(0xffffffffu, !ok)) break;
       tc_fence_after();
@@ -383,13 +402,7 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
                                   __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
           __syncwarp();
           const int wr = lane >> 3, wq = lane & 7;
-          float4 bq = make_float4(0.f, 0.f, 0.f, 0.f);
-          if (epi.bias) {
-            float bv[8];
-            Vec<bf16, 8>::load(static_cast<const bf16*>(epi.bias) + col + (wq & ~1) * 4, bv);
-            const int o = (wq & 1) * 4;
-            bq = make_float4(bv[o], bv[o + 1], bv[o + 2], bv[o + 3]);
-          }
+          const float4 bq = tc::bf16x4_to_f4(wbias);  // prefetched with the residual
           float4 cur[8];
           uint2 curg[8];
 #pragma unroll
@@ -427,6 +440,7 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
           for (int h = 0; h < 2; ++h)
 #pragma unroll
             for (int p = 0; p < 4; ++p) cur[h][p] = res[h][p];
+          const uint2 cbias[2] = {rbias[0], rbias[1]};  // prefetched with the residual
           if (c + 1 < c0 + CHUNKS) load_res(col + 32);  // prefetch the next chunk
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
@@ -437,13 +451,7 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
               srow[j] = make_float4(__uint_as_float(r[16 * h + 4 * j]), __uint_as_float(r[16 * h + 4 * j + 1]),
                                     __uint_as_float(r[16 * h + 4 * j + 2]), __uint_as_float(r[16 * h + 4 * j + 3]));
             __syncwarp();
-            float4 bq = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (epi.bias) {
-              float bv[8];
-              Vec<bf16, 8>::load(static_cast<const bf16*>(epi.bias) + col + h * 16 + (cq & ~1) * 4, bv);
-              const int o = (cq & 1) * 4;
-              bq = make_float4(bv[o], bv[o + 1], bv[o + 2], bv[o + 3]);
-            }
+            const float4 bq = tc::bf16x4_to_f4(cbias[h]);
 #pragma unroll
             for (int p = 0; p < 4; ++p) {
               const int lr = p * 8 + cr;
@@ -481,10 +489,20 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
               for (int i = 0; i < 8; ++i) v[8 * g + i] = fmaf(__uint_as_float(r[8 * g + i]), sv[i], bb[i]);
             }
           } else {
-            float bv[32];
-            if (epi.bias) Vec<bf16, 32>::load(static_cast<const bf16*>(epi.bias) + col, bv);
+            if (epi.bias) {
+              const uint32_t* bw = reinterpret_cast<const uint32_t*>(bpre);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]) + (epi.bias ? bv[i] : 0.f);
+              for (int i = 0; i < 16; ++i) {
+                const float2 b2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&bw[i]));
+                v[2 * i] = __uint_as_float(r[2 * i]) + b2.x;
+                v[2 * i + 1] = __uint_as_float(r[2 * i + 1]) + b2.y;
+              }
+            } else {
+#pragma unroll
+              for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+            }
+            // the next chunk's bias loads while this chunk is converted and stored
+            if (c + 1 < c0 + CHUNKS) load_bias(col + 32);
           }
           if (EK == tc::BF16OUT_SILU) {
 #pragma unroll
@@ -715,7 +733,9 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
   // proportionally less work per pipeline stage and runs well below the
   // BN = 256 rate. BN = 64 (153, on the line through the 128 and 256 points)
   // wins only when the 128-wide tiles fit in one round with SMs to spare: the
-  // few-row GEMMs of the diffusion head.
+  // few-row GEMMs of the diffusion head. The residual epilogue over long K
+  // has its own times (below), under which the full-layer fc2 (480 tiles of
+  // 256 in 4 rounds, or 640 of 192 in 5) takes the 192-wide tiles.
   int bn = 128;
   if (flags == 2 && N % 256 == 0) {
     bn = 256;
@@ -726,7 +746,12 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
   } else if (flags == 0) {
     const long mt = (M + tc::BM - 1) / tc::BM;
     long best = -1;
-    const int widths[4] = {256, 192, 128, 64}, tile_time[4] = {256, 243, 187, 153};
+    // The fp32-residual epilogue over long K (fc2) costs in proportion to the
+    // tile width: its measured round times at K = 3072 are 153 : 199 : 256.
+    const bool resid_half = epi.mode == LAZYMAR_EPI_RESIDUAL && !epi.gate && K >= 2048;
+    const int widths[4] = {256, 192, 128, 64};
+    const int tile_time_bf[4] = {256, 243, 187, 153}, tile_time_rh[4] = {256, 199, 153, 110};
+    const int* tile_time = resid_half ? tile_time_rh : tile_time_bf;
     for (int i = 0; i < 4; ++i) {
       if (N % widths[i] != 0) continue;
       const long rounds = (mt * (N / widths[i]) + c.num_sms - 1) / c.num_sms;
