@@ -387,12 +387,25 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
       const bool ok = mbar_wait(&acc_full[buf], use, abort_flag, err);
       if (__any_sync(0xffffffffu, !ok)) break;
       tc_fence_after();
+      // The tensor-memory load of chunk c + 1 is issued as soon as chunk c's
+      // accumulator registers have been consumed, and waited for at the top
+      // of the next iteration (the wait names the registers, so no use of
+      // them moves above it).
+      // (Only for the kinds where the extra live registers do not spill: the
+      // residual kind over short K and the bf16-output kinds up to 192 wide.
+      // The others load and wait at the top of each iteration.)
+      constexpr bool PIPE = EK == tc::RESID_WIDE || (tc::is_bf16out<EK>() && BN <= 192);
+      uint32_t r[32];
+      auto tld = [&](int c) {
+        tmem_ld32(tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN + c * 32), r);
+      };
+      if (PIPE) tld(c0);
 #pragma unroll 1
       for (int c = c0; c < c0 + CHUNKS; ++c) {
         const int col = n0 + c * 32;
-        uint32_t r[32];
-        tmem_ld32(tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN + c * 32), r);
-        tmem_wait_ld();
+        const bool more = c + 1 < c0 + CHUNKS;
+        if (!PIPE) tld(c);
+        tmem_wait_ld_regs(r);
         if (tc::is_wide<EK>()) {
           // whole 32-column fp32 chunk: 4 rows x 128 B per warp instruction
           float4* srow = reinterpret_cast<float4*>(stg + lane * C::STG_PITCH);
@@ -400,6 +413,7 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
           for (int j = 0; j < 8; ++j)
             srow[j] = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
                                   __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+          if (PIPE && more) tld(c + 1);
           __syncwarp();
           const int wr = lane >> 3, wq = lane & 7;
           const float4 bq = tc::bf16x4_to_f4(wbias);  // prefetched with the residual
@@ -517,6 +531,7 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
 #pragma unroll
             for (int i = 0; i < 16; ++i) w[i] = pack_bf16(v[2 * i], v[2 * i + 1]);
           }
+          if (PIPE && more) tld(c + 1);
           if (tma_out) {
             // the previous chunk's store must have read the staging buffer
             if (lane == 0) bulk_wait_read();
