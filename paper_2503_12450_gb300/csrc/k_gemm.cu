@@ -399,6 +399,13 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
       auto tld = [&](int c) {
         tmem_ld32(tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN + c * 32), r);
       };
+      // The tile's accumulator buffer goes back to the MMA warp as soon as
+      // this warp's last chunk is out of tensor memory, before its stores.
+      auto release = [&] {
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acc_empty[buf]);
+      };
       if (PIPE) tld(c0);
 #pragma unroll 1
       for (int c = c0; c < c0 + CHUNKS; ++c) {
@@ -414,6 +421,7 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
             srow[j] = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
                                   __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
           if (PIPE && more) tld(c + 1);
+          if (!more) release();  // the whole accumulator is out of tensor memory
           __syncwarp();
           const int wr = lane >> 3, wq = lane & 7;
           const float4 bq = tc::bf16x4_to_f4(wbias);  // prefetched with the residual
@@ -464,6 +472,7 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
             for (int j = 0; j < 4; ++j)
               srow[j] = make_float4(__uint_as_float(r[16 * h + 4 * j]), __uint_as_float(r[16 * h + 4 * j + 1]),
                                     __uint_as_float(r[16 * h + 4 * j + 2]), __uint_as_float(r[16 * h + 4 * j + 3]));
+            if (h == 1 && !more) release();
             __syncwarp();
             const float4 bq = tc::bf16x4_to_f4(cbias[h]);
 #pragma unroll
@@ -532,6 +541,7 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
             for (int i = 0; i < 16; ++i) w[i] = pack_bf16(v[2 * i], v[2 * i + 1]);
           }
           if (PIPE && more) tld(c + 1);
+          if (!more) release();
           if (tma_out) {
             // the previous chunk's store must have read the staging buffer
             if (lane == 0) bulk_wait_read();
@@ -565,9 +575,6 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
           }
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&acc_empty[buf]);
     }
     if (tma_out && lane == 0) bulk_wait_all();  // stores complete before the CTA exits
   }
