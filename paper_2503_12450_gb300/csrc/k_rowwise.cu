@@ -352,6 +352,36 @@ cudaError_t launch_cast(const Ctx& c, int dtype, const float* x, void* y, size_t
   return launch_pdl(cast_kernel<float>, dim3(grid), dim3(256), 0, c.stream, x, (float*)y, n);
 }
 
+// Gathers the selected tokens' query rows and residual rows into compact
+// buffers: row i of qc / xc is row row_map[i] of q / x. One CTA per row pair,
+// 16-byte vectors; q rows are D elements of TQ, x rows D fp32 values.
+template <typename TQ>
+__global__ void __launch_bounds__(128) gather_rows_kernel(const TQ* __restrict__ q, const float* __restrict__ x,
+                                                          const int* __restrict__ row_map, TQ* __restrict__ qc,
+                                                          float* __restrict__ xc, int D) {
+  pdl_wait();
+  pdl_trigger();
+  const size_t dst = blockIdx.x, src = (size_t)row_map[blockIdx.x];
+  const int nq = D * (int)sizeof(TQ) / 16, nx = D / 4;
+  const uint4* qs = reinterpret_cast<const uint4*>(q + src * D);
+  uint4* qd = reinterpret_cast<uint4*>(qc + dst * D);
+  const uint4* xs = reinterpret_cast<const uint4*>(x + src * D);
+  uint4* xd = reinterpret_cast<uint4*>(xc + dst * D);
+  for (int i = threadIdx.x; i < nq + nx; i += blockDim.x) {
+    if (i < nq) qd[i] = qs[i];
+    else xd[i - nq] = xs[i - nq];
+  }
+}
+cudaError_t launch_gather_rows(const Ctx& c, int dtype, const void* q, const float* x, const int* row_map, void* qc,
+                               float* xc, int M, int D) {
+  if (M == 0) return cudaSuccess;
+  if (dtype == LAZYMAR_BF16)
+    return launch_pdl(gather_rows_kernel<bf16>, dim3((unsigned)M), dim3(128), 0, c.stream, (const bf16*)q, x, row_map,
+                      (bf16*)qc, xc, D);
+  return launch_pdl(gather_rows_kernel<float>, dim3((unsigned)M), dim3(128), 0, c.stream, (const float*)q, x, row_map,
+                    (float*)qc, xc, D);
+}
+
 // ---------------------------------------------------------------------------
 // Classifier-free guidance with the condition cache
 // ---------------------------------------------------------------------------

@@ -496,12 +496,13 @@ lazymar_status layernorm(lazymar_handle* h, const Ctx& c, const float* x, const 
   });
 }
 
-lazymar_status attention(lazymar_handle* h, const Ctx& c, const void* k, const void* v, int rows, int n_q) {
+lazymar_status attention(lazymar_handle* h, const Ctx& c, const void* k, const void* v, int rows, int n_q,
+                         const void* q = nullptr) {
   if (rows == 0 || n_q == 0) return LAZYMAR_OK;
   const double flops = 4.0 * rows * n_q * (double)h->T * h->D;
   const double bytes = (double)h->es * h->D * (2.0 * rows * n_q + 2.0 * rows * h->T);
   return launch(h, LAZYMAR_K_ATTENTION, flops, bytes, c.stream, "attention", [&] {
-    return launch_attention(c, h->cfg.dtype, h->Q, k, v, h->O, rows, n_q, h->T, h->cfg.heads, h->dh);
+    return launch_attention(c, h->cfg.dtype, q ? q : h->Q, k, v, h->O, rows, n_q, h->T, h->cfg.heads, h->dh);
   });
 }
 
@@ -602,10 +603,25 @@ lazymar_status full_body(lazymar_handle* h, const Ctx& c, int B) {
 }
 
 // Device work of a cached step up to the output cache.
+//
+// Under the value criterion the output of block s-1 is read only for the
+// selected tokens (blocks s..L-1 see no other token's features, and the cache
+// keeps K/V of blocks >= s only). So block s-1 runs LN1 and the Q/K/V
+// projection over all tokens (its keys and values, and the value matrix Eq. 8
+// compares), then attention, out-projection and MLP for the selected tokens
+// alone. The feature criterion compares block s-1's output features, which
+// then run over all tokens.
 lazymar_status cached_body(lazymar_handle* h, const Ctx& c, int rows, int N, bool has_idx, int sel) {
   const int s = h->s, T = h->T, D = h->D;
+  const bool value = h->cfg.criterion == LAZYMAR_CRITERION_VALUE;
   LM_TRY(embed(h, c, rows, h->last_batch));
-  for (int l = 0; l < s; ++l) LM_TRY(layer_full(h, c, l, rows, h->Ks, h->Vs));
+  for (int l = 0; l < s - (value ? 1 : 0); ++l) LM_TRY(layer_full(h, c, l, rows, h->Ks, h->Vs));
+  if (value) {
+    const BlockDev& b = h->blk[s - 1];
+    const int M = rows * T;
+    LM_TRY(layernorm(h, c, h->H, nullptr, b.ln1_g, b.ln1_b, h->A, nullptr, M));
+    LM_TRY(gemm(h, c, h->A, b.w_qkv, M, 3 * D, D, GemmEpi{LAZYMAR_EPI_QKV, b.b_qkv, h->Q, D, h->Ks, h->Vs, nullptr, D}));
+  }
   // Eq. 8: similarity of block s-1's representation with the reference, then
   // the reference takes this step's values.
   const void* cur = h->Vs;
@@ -628,7 +644,21 @@ lazymar_status cached_body(lazymar_handle* h, const Ctx& c, int rows, int N, boo
                   }));
   }
   if (N > 0) {
-    for (int l = s; l < h->L; ++l) LM_TRY(layer_cached(h, c, l, rows, N, l == s));
+    if (value) {
+      // rest of block s-1 on the selected tokens: their queries and residual
+      // rows gathered (queries into the free LayerNorm buffer)
+      const BlockDev& b = h->blk[s - 1];
+      const int M = rows * N;
+      LM_TRY(launch(h, LAZYMAR_K_OTHER, 0, (double)M * D * (h->es + 4.0) * 2.0, c.stream, "gather", [&] {
+        return launch_gather_rows(c, h->cfg.dtype, h->Q, h->H, h->row_map, h->A, h->Hc, M, D);
+      }));
+      LM_TRY(attention(h, c, h->Ks, h->Vs, rows, N, h->A));
+      LM_TRY(gemm(h, c, h->O, b.w_o, M, D, D, GemmEpi{LAZYMAR_EPI_RESIDUAL, b.b_o, h->Hc, D, nullptr, nullptr, nullptr, D}));
+      LM_TRY(layernorm(h, c, h->Hc, nullptr, b.ln2_g, b.ln2_b, h->A, nullptr, M));
+      LM_TRY(gemm(h, c, h->A, b.w1, M, h->H4, D, GemmEpi{LAZYMAR_EPI_GELU, b.b1, h->U, h->H4, nullptr, nullptr, nullptr, D}));
+      LM_TRY(gemm(h, c, h->U, b.w2, M, D, h->H4, GemmEpi{LAZYMAR_EPI_RESIDUAL, b.b2, h->Hc, D, nullptr, nullptr, nullptr, D}));
+    }
+    for (int l = s; l < h->L; ++l) LM_TRY(layer_cached(h, c, l, rows, N, l == s && !value));
     LM_TRY(final_ln(h, c, h->Hc, h->row_map, rows * N));
   }
   return LAZYMAR_OK;

@@ -478,6 +478,9 @@ cudaError_t launch_embed(const Ctx& c, int dtype, const float* lat, const uint8_
                          float* H, int rows, int B, int T, int n_buffer, int n_img, int D, int token_dim,
                          int n_classes);
 cudaError_t launch_cast(const Ctx& c, int dtype, const float* x, void* y, size_t n);
+// Row i of qc / xc = row row_map[i] of q / x (D columns; D a multiple of 8).
+cudaError_t launch_gather_rows(const Ctx& c, int dtype, const void* q, const float* x, const int* row_map, void* qc,
+                               float* xc, int M, int D);
 // E4M3 copy of a bf16 weight matrix [rows, cols] with one scale per row
 // (max |w| / 448): q [rows, cols] bytes, scale [rows] fp32.
 cudaError_t launch_quantize_e4m3(const Ctx& c, const void* w, int rows, int cols, void* q, float* scale);
