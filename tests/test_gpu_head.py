@@ -163,3 +163,61 @@ def test_sampler_edge_shapes(td, steps, B, n_new):
     assert max_rel(got, want) < TOL["bf16"], max_rel(got, want)
     assert min_cos(got, want) >= COS_MIN
     h.close()
+
+
+def sampler_case(name, cond_dim, B, n_new, steps, max_tokens, seed):
+    torch_cuda()
+    n_img = 256
+    hc = S.head_config(name, n_steps=steps)
+    W = S.make_head_weights(hc, cond_dim, TD, seed=seed)
+    rng = np.random.default_rng(seed + 1)
+    z = S.round_bf16(rng.standard_normal((2 * B, n_img, cond_dim)).astype(np.float32))
+    pos = np.stack([rng.choice(n_img, n_new, replace=False) for _ in range(B)]).astype(np.int32)
+    h = lm.lazymar_head_create(hc, cond_dim, TD, W, max_tokens=max_tokens)
+    noise = S.make_head_noise(steps, B * n_new, TD, seed=seed + 2)
+    return hc, W, z, pos, noise, h
+
+
+@pytest.mark.parametrize("name,cond_dim,B,n_new,steps,max_tokens", [
+    ("mar_b", 768, 3, 50, 6, 150),     # 300 rows: three 128-row tiles, the last ragged
+    ("mar_l", 1024, 2, 5, 4, 10),      # width 1280, 8 blocks
+    ("mar_h", 1280, 2, 7, 3, 14),      # width 1536, 12 blocks
+    ("mar_b", 768, 2, 4, 100, 128),    # 100 kept steps whose modulations take two GEMMs (95 + 5 steps)
+])
+def test_sampler_widths_tiles_and_modulation_chunks(name, cond_dim, B, n_new, steps, max_tokens):
+    """The guided sampler at the MAR-B, MAR-L and MAR-H head widths, over
+    several ragged row tiles, and with the modulations of the kept steps
+    computed in two chunks, against the oracle."""
+    hc, W, z, pos, noise, h = sampler_case(name, cond_dim, B, n_new, steps, max_tokens, seed=71)
+    M = B * n_new
+    x = empty((M, TD))
+    lm.lazymar_head_sample(h, dev(z, "bf16"), B, 256, pos, n_new, noise, 3.0, 1.0, x)
+    lm.lazymar_head_sync(h)
+    zc, zu = z_rows(z, B, 256, pos)
+    want = HO.sample(W, HO.Schedule(hc["n_train"], steps), zc, zu, noise, 3.0, 1.0)
+    got = host(x)
+    assert max_rel(got, want) < TOL["bf16"], max_rel(got, want)
+    assert min_cos(got, want) >= COS_MIN
+    h.close()
+
+
+def test_sampler_graph_replay_is_bitwise_stable_at_mar_b_width():
+    """Eager, captured and replayed runs at width 1024 (tcgen05 block GEMMs)
+    give the same bits; a changed temperature is honoured by the replay."""
+    hc, W, z, pos, noise, h = sampler_case("mar_b", 768, 2, 6, 5, 12, seed=81)
+    zd = dev(z, "bf16")
+    outs = []
+    for _ in range(3):
+        x = empty((12, TD))
+        lm.lazymar_head_sample(h, zd, 2, 256, dev_int(pos), 6, dev(noise), 3.0, 1.0, x)
+        lm.lazymar_head_sync(h)
+        outs.append(host(x))
+    for o in outs[1:]:
+        assert np.array_equal(o, outs[0])
+    x = empty((12, TD))
+    lm.lazymar_head_sample(h, zd, 2, 256, dev_int(pos), 6, dev(noise), 3.0, 0.5, x)
+    lm.lazymar_head_sync(h)
+    zc, zu = z_rows(z, 2, 256, pos)
+    want = HO.sample(W, HO.Schedule(hc["n_train"], 5), zc, zu, noise, 3.0, 0.5)
+    assert max_rel(host(x), want) < TOL["bf16"]
+    h.close()
