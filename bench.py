@@ -525,7 +525,9 @@ def profile_case(args, cfg):
     N = synth.n_compute(cfg)
     dev = "cuda"
     if args.profile_case == "gemm_layers":
-        for M in (rows * T, rows * N, rows * N // 2):
+        # M: full blocks of both pathways, of the condition pathway alone, and
+        # the recomputed tokens of both / of the condition pathway
+        for M in (rows * T, rows * T // 2, rows * N, rows * N // 2):
             for n, k, epi in [(3 * D, D, lm.LAZYMAR_EPI_QKV), (D, D, lm.LAZYMAR_EPI_RESIDUAL),
                               (4 * D, D, lm.LAZYMAR_EPI_GELU), (D, 4 * D, lm.LAZYMAR_EPI_RESIDUAL)]:
                 a = torch.randn(M, k, device=dev).bfloat16()
