@@ -517,8 +517,9 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
 #pragma unroll
               for (int i = 0; i < 16; ++i) {
                 const float2 b2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&bw[i]));
-                v[2 * i] = __uint_as_float(r[2 * i]) + b2.x;
-                v[2 * i + 1] = __uint_as_float(r[2 * i + 1]) + b2.y;
+                f32x2_unpack(f32x2_add(f32x2_pack(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1])),
+                                       f32x2_pack(b2.x, b2.y)),
+                             v[2 * i], v[2 * i + 1]);
               }
             } else {
 #pragma unroll
@@ -532,7 +533,7 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
             for (int i = 0; i < 32; ++i) v[i] = silu(v[i]);
           } else if (epi.mode == LAZYMAR_EPI_GELU) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = gelu_erf(v[i]);
+            for (int i = 0; i < 16; ++i) gelu_erf_x2(v[2 * i], v[2 * i + 1]);
           }
           uint4 pk[4];
           {

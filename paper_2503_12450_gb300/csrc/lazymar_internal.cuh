@@ -114,6 +114,37 @@ __device__ __forceinline__ unsigned long long f32x2_add(unsigned long long a, un
   asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
   return d;
 }
+__device__ __forceinline__ unsigned long long f32x2_mul(unsigned long long a, unsigned long long b) {
+  unsigned long long d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
+// gelu_erf of two values with paired fp32 instructions, bit for bit the
+// scalar results: the polynomial runs in v = -u with the odd coefficients
+// negated (each Horner step is the scalar one with both operands negated, so
+// its rounding is the same), and -u h + (x + |x|) / 2 is the scalar fma.
+__device__ __forceinline__ void gelu_erf_x2(float& x0, float& x1) {
+  constexpr float kGeluP0 = -1.000018716e+00f;
+  constexpr float kGeluP1 = -1.150941610e+00f;
+  constexpr float kGeluP2 = -4.596132934e-01f;
+  constexpr float kGeluP3 = -5.220982432e-02f;
+  constexpr float kGeluP4 = 7.249599788e-03f;
+  constexpr float kGeluP5 = -4.984181724e-04f;
+  const float v0 = fmaxf(-fabsf(x0), -6.0f), v1 = fmaxf(-fabsf(x1), -6.0f);
+  const unsigned long long v = f32x2_pack(v0, v1);
+  unsigned long long p = f32x2_fma(f32x2_pack(-kGeluP5, -kGeluP5), v, f32x2_pack(kGeluP4, kGeluP4));
+  p = f32x2_fma(p, v, f32x2_pack(-kGeluP3, -kGeluP3));
+  p = f32x2_fma(p, v, f32x2_pack(kGeluP2, kGeluP2));
+  p = f32x2_fma(p, v, f32x2_pack(-kGeluP1, -kGeluP1));
+  p = f32x2_fma(p, v, f32x2_pack(kGeluP0, kGeluP0));
+  float p0, p1;
+  f32x2_unpack(p, p0, p1);
+  const unsigned long long h = f32x2_pack(exp2_approx(p0), exp2_approx(p1));
+  const unsigned long long half = f32x2_mul(f32x2_add(f32x2_pack(x0, x1), f32x2_pack(fabsf(x0), fabsf(x1))),
+                                            f32x2_pack(0.5f, 0.5f));
+  f32x2_unpack(f32x2_fma(v, h, half), x0, x1);
+}
 
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
