@@ -250,7 +250,11 @@ lazymar_status lazymar_cfg_combine(int dtype, int mode, const void *z_cond, cons
 
 /* Component entry points: the kernels the steps run, on caller buffers
  * (device pointers only), for parity tests and for callers composing their
- * own pipeline. */
+ * own pipeline. The kernels start while the previous kernel of the library on
+ * the same stream finishes (programmatic dependent launch) and wait for it
+ * before touching activations; weights (W of lazymar_linear, g and b of
+ * lazymar_layernorm) are read before that wait, so they must not be outputs
+ * of the library's kernel launched just before on the same stream. */
 
 /* y = a W^T + bias with a fused epilogue, a [M, K], W [N, K] (row-major,
  * dtype), bias [N] (dtype, may be NULL). bf16 runs on the tcgen05 tensor cores
@@ -292,7 +296,7 @@ lazymar_status lazymar_quantize_e4m3(const void *w, int rows, int cols, void *q,
 /* Multi-head bidirectional attention of Eq. 3 with a query subset: for each row
  * r and head h, O[r, j] = softmax(Q[r, j] K[r]^T / sqrt(dh)) V[r] over all T
  * keys. q, o: [rows, n_q, heads*head_dim]; k, v: [rows, T, heads*head_dim]
- * (dtype). bf16: head_dim 64 or 80, mma tensor cores with TMA-staged K/V. */
+ * (dtype). bf16: head_dim 64 or 80, tcgen05 tensor cores with TMA-staged K/V. */
 lazymar_status lazymar_attention(int dtype, const void *q, const void *k, const void *v, void *o,
                                  int rows, int n_q, int T, int heads, int head_dim, void *stream);
 

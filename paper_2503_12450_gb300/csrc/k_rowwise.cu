@@ -142,11 +142,33 @@ __device__ __forceinline__ void ln_stats(const float4 (&v)[NV], int D, float eps
   rstd = rsqrtf(warp_sum(q) / (float)D + eps);
 }
 
+// Four gain or shift values as loaded (packed bf16 or fp32). They are weights,
+// which no kernel writes, so the row kernels load them before waiting for the
+// predecessor grid.
+template <typename TO> struct Param4;
+template <> struct Param4<bf16> {
+  uint2 u;
+  __device__ __forceinline__ void load(const bf16* p) { u = *reinterpret_cast<const uint2*>(p); }
+  __device__ __forceinline__ float4 get() const {
+    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+    const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+    return make_float4(a.x, a.y, b.x, b.y);
+  }
+};
+template <> struct Param4<float> {
+  float4 u;
+  __device__ __forceinline__ void load(const float* p) { u = *reinterpret_cast<const float4*>(p); }
+  __device__ __forceinline__ float4 get() const { return u; }
+};
+
 template <typename TO>
-__device__ __forceinline__ void ln_write4(TO* y, const TO* g, const TO* b, int col, float4 x, float mean, float rstd) {
+__device__ __forceinline__ void ln_write4(TO* y, const Param4<TO>& gp, const Param4<TO>& bp, int col, float4 x,
+                                          float mean, float rstd) {
   float o[4] = {x.x, x.y, x.z, x.w};
+  const float4 g4 = gp.get(), b4 = bp.get();
+  const float gv[4] = {g4.x, g4.y, g4.z, g4.w}, bv[4] = {b4.x, b4.y, b4.z, b4.w};
 #pragma unroll
-  for (int k = 0; k < 4; ++k) o[k] = (o[k] - mean) * rstd * to_f(g[col + k]) + to_f(b[col + k]);
+  for (int k = 0; k < 4; ++k) o[k] = (o[k] - mean) * rstd * gv[k] + bv[k];
   if constexpr (sizeof(TO) == 2) {
     __nv_bfloat162 h0 = __floats2bfloat162_rn(o[0], o[1]), h1 = __floats2bfloat162_rn(o[2], o[3]);
     uint2 u;
@@ -163,9 +185,15 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const float* __restrict_
                                                         const TO* __restrict__ g, const TO* __restrict__ b,
                                                         TO* __restrict__ y, float* __restrict__ x_copy, int M, int D,
                                                         float eps) {
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  Param4<TO> gp[NV], bp[NV];
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    gp[i].load(g + 4 * (lane + 32 * i));
+    bp[i].load(b + 4 * (lane + 32 * i));
+  }
   pdl_wait();
   pdl_trigger();
-  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (row >= M) return;
   const int src = row_map ? row_map[row] : row;
   const float4* xr = reinterpret_cast<const float4*>(x + (size_t)src * D);
@@ -181,7 +209,7 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const float* __restrict_
   ln_stats<NV>(v, D, eps, mean, rstd);
   TO* yr = y + (size_t)row * D;
 #pragma unroll
-  for (int i = 0; i < NV; ++i) ln_write4<TO>(yr, g, b, 4 * (lane + 32 * i), v[i], mean, rstd);
+  for (int i = 0; i < NV; ++i) ln_write4<TO>(yr, gp[i], bp[i], 4 * (lane + 32 * i), v[i], mean, rstd);
 }
 
 // Four values to four E4M3 bytes (round to nearest even, saturating at the
@@ -200,9 +228,15 @@ __global__ void __launch_bounds__(256) layernorm_e4m3_kernel(const float* __rest
                                                              const TG* __restrict__ g, const TG* __restrict__ b,
                                                              uint8_t* __restrict__ y, float* __restrict__ x_copy,
                                                              int M, int D, float eps) {
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  Param4<TG> gp[NV], bp[NV];
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    gp[i].load(g + 4 * (lane + 32 * i));
+    bp[i].load(b + 4 * (lane + 32 * i));
+  }
   pdl_wait();
   pdl_trigger();
-  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (row >= M) return;
   const int src = row_map ? row_map[row] : row;
   const float4* xr = reinterpret_cast<const float4*>(x + (size_t)src * D);
@@ -220,7 +254,7 @@ __global__ void __launch_bounds__(256) layernorm_e4m3_kernel(const float* __rest
 #pragma unroll
   for (int i = 0; i < NV; ++i) {
     const int col = 4 * (lane + 32 * i);
-    const float4 gg = load4(g + col), bb = load4(b + col);
+    const float4 gg = gp[i].get(), bb = bp[i].get();
     *reinterpret_cast<uint32_t*>(yr + col) =
         pack_e4m3x4((v[i].x - mean) * rstd * gg.x + bb.x, (v[i].y - mean) * rstd * gg.y + bb.y,
                     (v[i].z - mean) * rstd * gg.z + bb.z, (v[i].w - mean) * rstd * gg.w + bb.w);
@@ -269,9 +303,15 @@ __global__ void __launch_bounds__(256) final_ln_kernel(const float* __restrict__
                                                        int T, int nb, int n_img, const TO* __restrict__ g,
                                                        const TO* __restrict__ b, TO* __restrict__ z, int M, int D,
                                                        float eps) {
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  Param4<TO> gp[NV], bp[NV];
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    gp[i].load(g + 4 * (lane + 32 * i));
+    bp[i].load(b + 4 * (lane + 32 * i));
+  }
   pdl_wait();
   pdl_trigger();
-  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (row >= M) return;
   const int tok = row_map ? row_map[row] : row;
   const int r = tok / T, t = tok - r * T;
@@ -284,7 +324,7 @@ __global__ void __launch_bounds__(256) final_ln_kernel(const float* __restrict__
   ln_stats<NV>(v, D, eps, mean, rstd);
   TO* zr = z + ((size_t)r * n_img + (t - nb)) * D;
 #pragma unroll
-  for (int i = 0; i < NV; ++i) ln_write4<TO>(zr, g, b, 4 * (lane + 32 * i), v[i], mean, rstd);
+  for (int i = 0; i < NV; ++i) ln_write4<TO>(zr, gp[i], bp[i], 4 * (lane + 32 * i), v[i], mean, rstd);
 }
 
 #define LM_LN_DISPATCH(KERNEL, TO, ...)                                                          \
