@@ -173,6 +173,15 @@ __global__ void __launch_bounds__(at2::THREADS, at2::Cfg<DH>::MIN_BLOCKS)
     for (int i = 0; i < N_BARS; ++i) mbar_init(&bars[i], (i == B_S_FREE || i == B_P_FULL) ? (uint32_t)n_act : 1u);
     *abort_flag = 0;
     fence_mbar_init();
+    // the descriptors are kernel parameters: fetched while the predecessor grid finishes
+    prefetch_tmap(&tmQ);
+    prefetch_tmap(&tmK);
+    prefetch_tmap(&tmV);
+    if (TAIL) {
+      prefetch_tmap(&tmQ2);
+      prefetch_tmap(&tmK2);
+      prefetch_tmap(&tmV2);
+    }
   }
   if (warp == 4) {
     tmem_alloc(tmem_slot, C::TMEM_COLS);

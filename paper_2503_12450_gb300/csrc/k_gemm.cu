@@ -216,6 +216,13 @@ __global__ void __launch_bounds__(tc::Cfg<BN, EK, BK, F8>::THREADS, 1)
     fence_mbar_init();
     prefetch_tmap(&tmA);
     prefetch_tmap(&tmB);
+    if (tma_out) {
+      prefetch_tmap(&tmO0);
+      if (epi.mode == LAZYMAR_EPI_QKV) {
+        prefetch_tmap(&tmO1);
+        prefetch_tmap(&tmO2);
+      }
+    }
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, C::TMEM_COLS);
