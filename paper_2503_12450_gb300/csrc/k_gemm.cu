@@ -749,49 +749,58 @@ static cudaError_t launch_tc(const Ctx& c, const void* A, const void* W, int M, 
                     epi, c.err);
 }
 
-cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, int M, int N, int K,
-                        const GemmEpi& epi, int flags) {
-  if (M == 0) return cudaSuccess;
-  if (dtype == LAZYMAR_F32) {
-    dim3 grid((N + 63) / 64, (M + 63) / 64);
-    return launch_pdl(gemm_f32_kernel, grid, dim3(256), 0, c.stream, static_cast<const float*>(A),
-                      static_cast<const float*>(W), M, N, K, epi);
-  }
-  // Tile width: the one with the fewest rounds of tiles over the SMs x the
-  // time of one tile. Relative tile times 187 : 243 : 256 for BN = 128 : 192 :
-  // 256 (measured, one round of 128 x BN x 3072 tiles): a narrower tile does
-  // proportionally less work per pipeline stage and runs well below the
-  // BN = 256 rate. BN = 64 (153, on the line through the 128 and 256 points)
-  // wins only when the 128-wide tiles fit in one round with SMs to spare: the
-  // few-row GEMMs of the diffusion head. The residual epilogue over long K
-  // has its own times (below), under which the full-layer fc2 (480 tiles of
-  // 256 in 4 rounds, or 640 of 192 in 5) takes the 192-wide tiles.
+// Relative time of one round of tiles of width bn (see launch_gemm).
+static int tile_time(int bn, bool resid_half) {
+  static const int widths[4] = {256, 192, 128, 64};
+  static const int t_bf[4] = {256, 243, 187, 153}, t_rh[4] = {256, 199, 153, 110};
+  for (int i = 0; i < 4; ++i)
+    if (widths[i] == bn) return resid_half ? t_rh[i] : t_bf[i];
+  return 256;
+}
+
+// Tile width with the fewest rounds of tiles over the SMs x the time of one
+// tile, and that cost.
+static int choose_bn(const Ctx& c, int M, int N, const GemmEpi& epi, int K, long* cost) {
+  const long mt = (M + tc::BM - 1) / tc::BM;
+  const bool resid_half = epi.mode == LAZYMAR_EPI_RESIDUAL && !epi.gate && K >= 2048;
+  const int widths[4] = {256, 192, 128, 64};
   int bn = 128;
-  if (flags == 2 && N % 256 == 0) {
-    bn = 256;
-  } else if (flags == 3 && N % 192 == 0) {
-    bn = 192;
-  } else if (flags == 4) {
-    bn = 64;
-  } else if (flags == 0) {
-    const long mt = (M + tc::BM - 1) / tc::BM;
-    long best = -1;
-    // The fp32-residual epilogue over long K (fc2) costs in proportion to the
-    // tile width: its measured round times at K = 3072 are 153 : 199 : 256.
-    const bool resid_half = epi.mode == LAZYMAR_EPI_RESIDUAL && !epi.gate && K >= 2048;
-    const int widths[4] = {256, 192, 128, 64};
-    const int tile_time_bf[4] = {256, 243, 187, 153}, tile_time_rh[4] = {256, 199, 153, 110};
-    const int* tile_time = resid_half ? tile_time_rh : tile_time_bf;
-    for (int i = 0; i < 4; ++i) {
-      if (N % widths[i] != 0) continue;
-      const long rounds = (mt * (N / widths[i]) + c.num_sms - 1) / c.num_sms;
-      const long cost = rounds * tile_time[i];
-      if (best < 0 || cost < best) {
-        best = cost;
-        bn = widths[i];
-      }
+  long best = -1;
+  for (int i = 0; i < 4; ++i) {
+    if (N % widths[i] != 0) continue;
+    const long rounds = (mt * (N / widths[i]) + c.num_sms - 1) / c.num_sms;
+    const long t = rounds * tile_time(widths[i], resid_half);
+    if (best < 0 || t < best) {
+      best = t;
+      bn = widths[i];
     }
   }
+  *cost = best;
+  return bn;
+}
+
+// The epilogue of rows [m0, M) of a GEMM as a GEMM of its own.
+static GemmEpi epi_from_row(const GemmEpi& e, int m0) {
+  GemmEpi t = e;
+  if (e.mode == LAZYMAR_EPI_QKV) {
+    t.out = static_cast<bf16*>(e.out) + (size_t)m0 * e.D;
+    if (e.row_map) {
+      t.row_map = e.row_map + m0;
+    } else {
+      t.k_out = static_cast<bf16*>(e.k_out) + (size_t)m0 * e.D;
+      t.v_out = static_cast<bf16*>(e.v_out) + (size_t)m0 * e.D;
+    }
+  } else if (e.mode == LAZYMAR_EPI_RESIDUAL) {
+    t.out = static_cast<float*>(e.out) + (size_t)m0 * e.ldo;
+    if (e.gate) t.gate = static_cast<const bf16*>(e.gate) + (size_t)m0 * e.ldg;
+  } else {
+    t.out = static_cast<bf16*>(e.out) + (size_t)m0 * e.ldo;
+  }
+  return t;
+}
+
+static cudaError_t launch_bn(const Ctx& c, int dtype, const void* A, const void* W, int M, int N, int K,
+                             const GemmEpi& epi, int bn) {
   if (dtype == LAZYMAR_E4M3) {
     // E4M3 operands (bf16-output kinds): a 128-element stage is one atom; the
     // tile width follows the bf16 choice
@@ -844,6 +853,64 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
   if (ek == tc::RESID_HALF) return launch_tc<128, tc::RESID_HALF, 64>(c, A, W, M, N, K, epi);
   if (ek == tc::BF16OUT_SILU) return launch_tc<128, tc::BF16OUT_SILU, 64>(c, A, W, M, N, K, epi);
   return launch_tc<128, tc::BF16OUT, 64>(c, A, W, M, N, K, epi);
+}
+
+
+
+cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, int M, int N, int K,
+                        const GemmEpi& epi, int flags) {
+  if (M == 0) return cudaSuccess;
+  if (dtype == LAZYMAR_F32) {
+    dim3 grid((N + 63) / 64, (M + 63) / 64);
+    return launch_pdl(gemm_f32_kernel, grid, dim3(256), 0, c.stream, static_cast<const float*>(A),
+                      static_cast<const float*>(W), M, N, K, epi);
+  }
+  // Tile width: the one with the fewest rounds of tiles over the SMs x the
+  // time of one tile. Relative tile times 187 : 243 : 256 for BN = 128 : 192 :
+  // 256 (measured, one round of 128 x BN x 3072 tiles): a narrower tile does
+  // proportionally less work per pipeline stage and runs well below the
+  // BN = 256 rate. BN = 64 (153, on the line through the 128 and 256 points)
+  // wins only when the 128-wide tiles fit in one round with SMs to spare: the
+  // few-row GEMMs of the diffusion head. The fp32-residual epilogue over long K
+  // (fc2) costs in proportion to the tile width: its measured round times at
+  // K = 3072 are 153 : 199 : 256 (110 for 64), under which the full-layer fc2
+  // (480 tiles of 256 in 4 rounds, or 640 of 192 in 5) takes the 192-wide tiles.
+  if (flags == 2 && N % 256 == 0) return launch_bn(c, dtype, A, W, M, N, K, epi, 256);
+  if (flags == 3 && N % 192 == 0) return launch_bn(c, dtype, A, W, M, N, K, epi, 192);
+  if (flags == 4) return launch_bn(c, dtype, A, W, M, N, K, epi, 64);
+  if (flags != 0) return launch_bn(c, dtype, A, W, M, N, K, epi, 128);
+  long cost = 0;
+  const int bn = choose_bn(c, M, N, epi, K, &cost);
+  // Last-wave split of the fp32-residual GEMM over short K (the
+  // out-projection): when its tiles fill several rounds but the last one only
+  // partly, the row tiles of the whole waves run as one launch and the
+  // remaining rows as a second launch, with the tile width that suits their
+  // count (narrower tiles spread them over all SMs), if the model puts the
+  // pair at least 2 % below the one launch. Measured on the MAR-B full layer:
+  // the partial fourth round of 256-wide tiles costs a whole round (8.2 us),
+  // while the last 8 row tiles as 64-wide tiles take 4.9 us (34.1 -> 30.9
+  // us). The other kinds lose: the residual over long K (fc2) runs its partial
+  // last round faster than a full one (32 tiles of 192 in 10.8 us against
+  // 17.1 us), and the full-layer Q/K/V went 55.9 -> 57.6 us split.
+  if (dtype == LAZYMAR_BF16 && epi.mode == LAZYMAR_EPI_RESIDUAL && !epi.gate && K < 2048) {
+    const long mt = (M + tc::BM - 1) / tc::BM, nn = N / bn;
+    const long rounds = (mt * nn + c.num_sms - 1) / c.num_sms;
+    const long body_rt = rounds >= 3 ? (rounds - 1) * c.num_sms / nn : 0;  // whole row tiles of the full waves
+    if (body_rt > 0 && body_rt < mt) {
+      const int Mb = (int)(body_rt * tc::BM);
+      long tail_cost = 0;
+      const int tail_bn = choose_bn(c, M - Mb, N, epi, K, &tail_cost);
+      const long body_rounds = (body_rt * nn + c.num_sms - 1) / c.num_sms;
+      const long split_cost = body_rounds * tile_time(bn, false) + tail_cost;
+      if (split_cost * 50 <= cost * 49) {
+        const cudaError_t e = launch_bn(c, dtype, A, W, Mb, N, K, epi, bn);
+        if (e != cudaSuccess) return e;
+        return launch_bn(c, dtype, static_cast<const bf16*>(A) + (size_t)Mb * K, W, M - Mb, N, K,
+                         epi_from_row(epi, Mb), tail_bn);
+      }
+    }
+  }
+  return launch_bn(c, dtype, A, W, M, N, K, epi, bn);
 }
 
 }  // namespace lm

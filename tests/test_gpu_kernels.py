@@ -207,7 +207,7 @@ GEMM_SHAPES = [
 ]
 
 
-def _linear_case(dtype, epi, M, N, K, flags, seed):
+def _linear_case(dtype, epi, M, N, K, flags, seed, scatter=True):
     torch = torch_cuda()
     a = synth.tensor((M, K), seed, dtype=dtype)
     w = synth.tensor((N, K), seed + 1, std=0.05, dtype=dtype)
@@ -227,6 +227,14 @@ def _linear_case(dtype, epi, M, N, K, flags, seed):
         lm.lazymar_linear(DT[dtype], epi, ga, gw, gb, M, N, K, out, N, flags=flags)
         sync()
         assert max_rel(host(out), r0 + ref) < 1e-4
+    elif not scatter:
+        D = N // 3
+        q, gk, gv = empty((M, D), dtype), empty((M, D), dtype), empty((M, D), dtype)
+        lm.lazymar_linear(DT[dtype], epi, ga, gw, gb, M, N, K, q, D, gk, gv, None, flags=flags)
+        sync()
+        assert max_rel(host(q), ref[:, :D]) < out_dtype_tol
+        assert max_rel(host(gk), ref[:, D:2 * D]) < out_dtype_tol
+        assert max_rel(host(gv), ref[:, 2 * D:]) < out_dtype_tol
     else:
         D = N // 3
         R = M + 17
@@ -252,6 +260,21 @@ def test_linear_bf16_tcgen05(M, N, K, epi):
         pytest.skip("not a QKV shape")
     for flags in [1, 4] + ([2] if N % 256 == 0 else []) + ([3] if N % 192 == 0 else []):
         _linear_case("bf16", epi, M, N, K, flags, seed=M + N + K + epi)
+
+
+@pytest.mark.parametrize("M,N,K,epi", [
+    (20480, 768, 768, lm.LAZYMAR_EPI_RESIDUAL),    # out-projection: three waves of 256-wide tiles, then 8 row tiles 64 wide
+    (20480, 768, 3072, lm.LAZYMAR_EPI_RESIDUAL),   # residual over long K (fc2): one launch
+    (20480, 2304, 768, lm.LAZYMAR_EPI_QKV),        # other epilogues: one launch
+])
+def test_linear_last_wave_split(M, N, K, epi):
+    """With the automatic tile width (flags 0) the fp32-residual GEMM over
+    short K whose last round of tiles would run mostly empty is launched as
+    two: the row tiles of the whole waves, then the remaining rows (their A
+    rows and residual rows offset) with narrower tiles."""
+    _linear_case("bf16", epi, M, N, K, 0, seed=M + N + K + epi)
+    if epi == lm.LAZYMAR_EPI_QKV:
+        _linear_case("bf16", epi, M, N, K, 0, seed=M + N + K, scatter=False)
 
 
 @pytest.mark.parametrize("M,N,K", [(1, 12, 8), (40, 768, 256), (160, 1024, 256), (77, 256, 1024)])
