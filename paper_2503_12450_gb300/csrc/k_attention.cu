@@ -286,8 +286,15 @@ __global__ void __launch_bounds__(at2::THREADS, at2::Cfg<DH>::MIN_BLOCKS)
       // row max of the raw scores; keys beyond T (the last chunk only) drop out
       float mloc = -FLT_MAX;
       if (c * KC + KC <= T) {
+        // four independent chains of three-input maxima (dependency depth 8
+        // instead of 32)
+        float mq[4] = {-FLT_MAX, -FLT_MAX, -FLT_MAX, -FLT_MAX};
 #pragma unroll
-        for (int i = 0; i < 64; i += 2) mloc = fmax3(mloc, sv[i], sv[i + 1]);
+        for (int i = 0; i < 64; i += 8) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q) mq[q] = fmax3(mq[q], sv[i + 2 * q], sv[i + 2 * q + 1]);
+        }
+        mloc = fmax3(mq[0], mq[1], fmaxf(mq[2], mq[3]));
       } else {
 #pragma unroll
         for (int i = 0; i < 64; ++i) {
@@ -308,18 +315,20 @@ __global__ void __launch_bounds__(at2::THREADS, at2::Cfg<DH>::MIN_BLOCKS)
       // exponent arguments and the row sum two keys per instruction (the
       // softmax is bound by instruction issue)
       const unsigned long long sc2 = f32x2_pack(scale_log2, scale_log2), nm2 = f32x2_pack(-m_run, -m_run);
-      unsigned long long ps2 = f32x2_pack(0.f, 0.f);
+      // the row sum in four independent paired accumulators
+      unsigned long long ps2[4] = {f32x2_pack(0.f, 0.f), f32x2_pack(0.f, 0.f), f32x2_pack(0.f, 0.f),
+                                   f32x2_pack(0.f, 0.f)};
       uint32_t pk[32];
 #pragma unroll
       for (int i = 0; i < 32; ++i) {
         float x0, x1;
         f32x2_unpack(f32x2_fma(f32x2_pack(sv[2 * i], sv[2 * i + 1]), sc2, nm2), x0, x1);
         const float p0 = exp2_approx(x0), p1 = exp2_approx(x1);
-        ps2 = f32x2_add(ps2, f32x2_pack(p0, p1));
+        ps2[i & 3] = f32x2_add(ps2[i & 3], f32x2_pack(p0, p1));
         pk[i] = pack_bf16(p0, p1);
       }
       float ps0, ps1;
-      f32x2_unpack(ps2, ps0, ps1);
+      f32x2_unpack(f32x2_add(f32x2_add(ps2[0], ps2[1]), f32x2_add(ps2[2], ps2[3])), ps0, ps1);
       const float psum = ps0 + ps1;
       // PV(c-1) must be complete before O is rescaled or P is overwritten.
       if (c > 0) {
