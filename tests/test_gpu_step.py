@@ -533,3 +533,27 @@ def test_graph_replay_matches_eager_execution():
     assert np.array_equal(host(zz), z1)
     np.testing.assert_allclose(host(gg), z1[:r.B], rtol=1e-2, atol=1e-6)   # gamma = 1: guided = c
     r.h.close()
+
+
+@pytest.mark.parametrize("name,reuse", [("mar_b", False), ("mar_b", True), ("mar_h", True)])
+def test_full_recompute_cached_step_equals_full_step_bf16(name, reuse):
+    """A cached step that recomputes all T tokens is a full step (the
+    oracle's invariant, at full batch and bf16): block s-1 gathers every
+    token, the compact GEMMs run at M = rows T (the out-projection as two
+    launches), and the features and guided output match the full step's
+    within the bf16 bar; with the condition cache reused the conditional
+    rows alone run."""
+    r = Run(name)
+    T = r.T
+    st0, st1 = r.state(100), r.state(104)
+    r.full(st0)
+    zf, gf = r.full(st1)
+    r.full(st0)
+    zc, gc, I = r.cached(st1, T, reuse)
+    rows = r.B if reuse else 2 * r.B
+    assert I.shape == (rows, T) and (I == np.arange(T)).all()
+    assert max_rel(zc[:r.B], zf[:r.B]) < TOL["bf16"] and min_cos(zc[:r.B], zf[:r.B]) >= COS_MIN
+    if not reuse:
+        assert max_rel(zc, zf) < TOL["bf16"] and min_cos(zc, zf) >= COS_MIN
+        for b in (0, r.B - 1):
+            assert guided_ok(gc[b], gf[b], zf[pair_rows(r.B, b)], GAMMA, TOL["bf16"])
