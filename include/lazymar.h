@@ -443,9 +443,11 @@ lazymar_status lazymar_head_sync(lazymar_head *hd, void *stream);
  * Returns INVALID_ARG unless 1 <= n_steps <= n_train. */
 lazymar_status lazymar_head_schedule(int n_train, int n_steps, int32_t *kept, float *consts);
 
-/* Per kernel class: launches, algorithmic flops and bytes, and (while
- * profiling is on) device time from CUDA events recorded around each launch on
- * its stream. lazymar_get_stats waits for the recorded events. */
+/* Per kernel class: kernel launches (a GEMM split into two launches counts
+ * two), algorithmic flops and bytes, and (while profiling is on) device time
+ * from CUDA events recorded around each call on its stream (timed_launches
+ * counts those event pairs; one pair encloses both launches of a split GEMM).
+ * lazymar_get_stats waits for the recorded events. */
 enum {
   LAZYMAR_K_GEMM = 0, LAZYMAR_K_ATTENTION = 1, LAZYMAR_K_LAYERNORM = 2, LAZYMAR_K_SELECT = 3,
   LAZYMAR_K_EMBED = 4, LAZYMAR_K_CFG = 5, LAZYMAR_K_OTHER = 6, LAZYMAR_K_COUNT = 7

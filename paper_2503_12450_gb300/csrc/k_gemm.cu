@@ -799,8 +799,21 @@ static GemmEpi epi_from_row(const GemmEpi& e, int m0) {
   return t;
 }
 
+// Kernels issued by launch_gemm on this thread (a last-wave split issues two).
+static thread_local long long t_gemm_kernels = 0;
+long long gemm_kernels_issued() { return t_gemm_kernels; }
+
+static cudaError_t launch_bn_impl(const Ctx& c, int dtype, const void* A, const void* W, int M, int N, int K,
+                                  const GemmEpi& epi, int bn);
 static cudaError_t launch_bn(const Ctx& c, int dtype, const void* A, const void* W, int M, int N, int K,
                              const GemmEpi& epi, int bn) {
+  const cudaError_t e = launch_bn_impl(c, dtype, A, W, M, N, K, epi, bn);
+  if (e == cudaSuccess) ++t_gemm_kernels;
+  return e;
+}
+
+static cudaError_t launch_bn_impl(const Ctx& c, int dtype, const void* A, const void* W, int M, int N, int K,
+                                  const GemmEpi& epi, int bn) {
   if (dtype == LAZYMAR_E4M3) {
     // E4M3 operands (bf16-output kinds): a 128-element stage is one atom; the
     // tile width follows the bf16 choice
@@ -862,8 +875,10 @@ cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, i
   if (M == 0) return cudaSuccess;
   if (dtype == LAZYMAR_F32) {
     dim3 grid((N + 63) / 64, (M + 63) / 64);
-    return launch_pdl(gemm_f32_kernel, grid, dim3(256), 0, c.stream, static_cast<const float*>(A),
-                      static_cast<const float*>(W), M, N, K, epi);
+    const cudaError_t e = launch_pdl(gemm_f32_kernel, grid, dim3(256), 0, c.stream, static_cast<const float*>(A),
+                                     static_cast<const float*>(W), M, N, K, epi);
+    if (e == cudaSuccess) ++t_gemm_kernels;
+    return e;
   }
   // Tile width: the one with the fewest rounds of tiles over the SMs x the
   // time of one tile. Relative tile times 187 : 243 : 256 for BN = 128 : 192 :

@@ -482,8 +482,13 @@ lazymar_status gemm(lazymar_handle* h, const Ctx& c, const void* A, const void* 
   const int dt = dtype < 0 ? h->cfg.dtype : dtype;
   double bytes = gemm_bytes(h, M, N, K, e.mode);
   if (dt == LAZYMAR_E4M3) bytes -= (double)h->es * ((double)M * K + (double)N * K) / 2.0;  // 1-byte operands
-  return launch(h, LAZYMAR_K_GEMM, 2.0 * M * N * K, bytes, c.stream, "gemm",
-                [&] { return launch_gemm(c, dt, A, W, M, N, K, e, 0); });
+  const long long k0 = gemm_kernels_issued();
+  LM_TRY(launch(h, LAZYMAR_K_GEMM, 2.0 * M * N * K, bytes, c.stream, "gemm",
+                [&] { return launch_gemm(c, dt, A, W, M, N, K, e, 0); }));
+  // the statistics count kernels: a split GEMM adds its second launch
+  const long long extra = gemm_kernels_issued() - k0 - 1;
+  if (extra > 0) h->stats.k[LAZYMAR_K_GEMM].launches += extra;
+  return LAZYMAR_OK;
 }
 
 lazymar_status layernorm(lazymar_handle* h, const Ctx& c, const float* x, const int* map, const void* g, const void* b,

@@ -488,6 +488,9 @@ struct GemmEpi {
 };
 cudaError_t launch_gemm(const Ctx& c, int dtype, const void* A, const void* W, int M, int N, int K,
                         const GemmEpi& epi, int flags);
+// Running count of the GEMM kernels launch_gemm has issued on this thread
+// (a GEMM split into two launches counts two).
+long long gemm_kernels_issued();
 // Checks the preconditions of launch_gemm; returns false with a message.
 bool gemm_supported(int dtype, int M, int N, int K, const GemmEpi& epi, const char** why);
 
