@@ -203,12 +203,17 @@ __global__ void __launch_bounds__(FIN_THREADS, 2) final_kernel(const float* __re
   float* h = sm;                        // [2][w] modulated rows
   float* o = sm + 2 * w;                // [2][2 td] outputs
   float* red = o + 4 * td;              // [2][FIN_THREADS / 32] partial sums
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  constexpr int NWARP = FIN_THREADS / 32;
+  // The output weights (no kernel writes them) of this warp's output columns
+  // oc = warp + 8 i go to L1 while the predecessor grid finishes.
+  for (int oc = warp; oc < 2 * td; oc += NWARP)
+    for (int c = 8 * lane; c < w; c += 256)
+      asm volatile("prefetch.global.L1 [%0];" ::"l"(wout + (size_t)oc * w + c));
   pdl_wait();
   pdl_trigger();
   const int m = blockIdx.x;
   if (m >= M) return;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  constexpr int NW = FIN_THREADS / 32;
   // both rows at once: threads 0-127 normalise row m (conditional), threads
   // 128-255 row M + m (unconditional); each thread holds w / 128 <= 16
   // columns t + 128 i, and the modulation loads go out with the row's
@@ -242,38 +247,50 @@ __global__ void __launch_bounds__(FIN_THREADS, 2) final_kernel(const float* __re
         q = fmaf(d, d, q);
       }
     q = warp_sum(q);
-    if (lane == 0) red[NW + warp] = q;
+    if (lane == 0) red[NWARP + warp] = q;
     __syncthreads();
-    const float qt = (red[NW + 4 * g] + red[NW + 4 * g + 1]) + (red[NW + 4 * g + 2] + red[NW + 4 * g + 3]);
+    const float qt = (red[NWARP + 4 * g] + red[NWARP + 4 * g + 1]) + (red[NWARP + 4 * g + 2] + red[NWARP + 4 * g + 3]);
     const float rstd = rsqrtf(qt / (float)w + eps);
 #pragma unroll
     for (int i = 0; i < 16; ++i)
       if (i < n) h[g * w + t + 128 * i] = fmaf((v[i] - mean) * rstd, 1.f + scl[i], sh[i]);
     __syncthreads();
   }
-  // 2 rows x 2 td outputs, one warp per output at a time; each lane takes 8
-  // consecutive columns per 256 (one 16-byte weight load, w % 128 == 0)
-  for (int k = warp; k < 4 * td; k += NW) {
-    const int s = k / (2 * td), oc = k - s * 2 * td;
-    const bf16* wr = wout + (size_t)oc * w;
-    const float* hs = h + s * w;
-    float acc0 = 0.f, acc1 = 0.f;
+  // 2 rows x 2 td outputs: warp w takes output columns oc = w + 8 i, two at a
+  // time, each for both rows (one weight load serves two rows); each lane
+  // takes 8 consecutive columns per 256 (one 16-byte weight load, w % 128 == 0)
+  for (int oa = warp; oa < 2 * td; oa += 2 * NWARP) {
+    const int ob = oa + NWARP;
+    const bool two = ob < 2 * td;
+    const bf16* wa = wout + (size_t)oa * w;
+    const bf16* wb = wout + (size_t)(two ? ob : oa) * w;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};  // (oa, row 0), (oa, row 1), (ob, row 0), (ob, row 1)
     for (int c = 8 * lane; c < w; c += 256) {
-      float wv[8];
-      Vec<bf16, 8>::load(wr + c, wv);
-      const float4 h0 = *reinterpret_cast<const float4*>(hs + c);
-      const float4 h1 = *reinterpret_cast<const float4*>(hs + c + 4);
-      acc0 = fmaf(h0.x, wv[0], acc0);
-      acc1 = fmaf(h0.y, wv[1], acc1);
-      acc0 = fmaf(h0.z, wv[2], acc0);
-      acc1 = fmaf(h0.w, wv[3], acc1);
-      acc0 = fmaf(h1.x, wv[4], acc0);
-      acc1 = fmaf(h1.y, wv[5], acc1);
-      acc0 = fmaf(h1.z, wv[6], acc0);
-      acc1 = fmaf(h1.w, wv[7], acc1);
+      float va[8], vb[8];
+      Vec<bf16, 8>::load(wa + c, va);
+      Vec<bf16, 8>::load(wb + c, vb);
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        const float4 h0 = *reinterpret_cast<const float4*>(h + r * w + c);
+        const float4 h1 = *reinterpret_cast<const float4*>(h + r * w + c + 4);
+        const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          acc[r] = fmaf(hv[e], va[e], acc[r]);
+          acc[2 + r] = fmaf(hv[e], vb[e], acc[2 + r]);
+        }
+      }
     }
-    const float acc = warp_sum(acc0 + acc1);
-    if (lane == 0) o[k] = acc + bout[oc];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) acc[i] = warp_sum(acc[i]);
+    if (lane == 0) {
+      o[oa] = acc[0] + bout[oa];
+      o[2 * td + oa] = acc[1] + bout[oa];
+      if (two) {
+        o[ob] = acc[2] + bout[ob];
+        o[2 * td + ob] = acc[3] + bout[ob];
+      }
+    }
   }
   __syncthreads();
   if (eval_out) {
