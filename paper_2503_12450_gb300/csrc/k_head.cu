@@ -97,25 +97,19 @@ __global__ void __launch_bounds__(256) cond_silu_kernel(const bf16* __restrict__
   }
 }
 
-// One warp per row, VPL float4 per lane (w = 128 VPL): the row's LayerNorm
-// without gain or shift, modulated by (1 + scale) and shift from the mod row,
-// to bf16. With INPROJ the row is first computed as W_in x + b_in from the
-// token's latent (x row m = r mod M; W_in stored transposed, [td, w]).
+// One row by one warp, VPL float4 per lane (w = 128 VPL): the row's
+// LayerNorm without gain or shift, modulated by (1 + scale) and shift from
+// the modulation row mr, to bf16 at hr. With INPROJ the row is first computed
+// as W_in x + b_in from the token's latent xm (W_in stored transposed,
+// [td, w]) and stored to xr; otherwise it is read from xr.
 template <int VPL, bool INPROJ>
-__global__ void __launch_bounds__(256) ln_mod_kernel(float* __restrict__ xh, const float* __restrict__ x,
-                                                     const bf16* __restrict__ win_t, const bf16* __restrict__ bin,
-                                                     const bf16* __restrict__ mod, int ldm, int shift_off,
-                                                     int scale_off, bf16* __restrict__ hb, int R, int M, int td,
-                                                     float eps) {
-  pdl_wait();
-  pdl_trigger();
-  const int r = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
-  if (r >= R) return;
+__device__ __forceinline__ void ln_mod_row(float* __restrict__ xr, const float* __restrict__ xm,
+                                           const bf16* __restrict__ win_t, const bf16* __restrict__ bin,
+                                           const bf16* __restrict__ mr, int shift_off, int scale_off,
+                                           bf16* __restrict__ hr, int td, float eps, int lane) {
   constexpr int w = 128 * VPL;
   float4 v[VPL];
-  float* xr = xh + (size_t)r * w;
   // the modulation does not depend on the row: its loads go out first
-  const bf16* mr = mod + (size_t)r * ldm;
   uint2 shp[VPL], scp[VPL];
 #pragma unroll
   for (int i = 0; i < VPL; ++i) {
@@ -125,7 +119,6 @@ __global__ void __launch_bounds__(256) ln_mod_kernel(float* __restrict__ xh, con
   }
   if (INPROJ) {
     // latent index k outermost: each k issues VPL independent weight loads
-    const float* xm = x + (size_t)(r < M ? r : r - M) * td;
 #pragma unroll
     for (int i = 0; i < VPL; ++i) {
       float a[4];
@@ -176,8 +169,25 @@ __global__ void __launch_bounds__(256) ln_mod_kernel(float* __restrict__ xh, con
     uint2 u;
     u.x = pack_bf16(o0, o1);
     u.y = pack_bf16(o2, o3);
-    *reinterpret_cast<uint2*>(hb + (size_t)r * w + c) = u;
+    *reinterpret_cast<uint2*>(hr + c) = u;
   }
+}
+
+// One warp per row r of R (ln_mod_row; with INPROJ from the latent of
+// token r mod M).
+template <int VPL, bool INPROJ>
+__global__ void __launch_bounds__(256) ln_mod_kernel(float* __restrict__ xh, const float* __restrict__ x,
+                                                     const bf16* __restrict__ win_t, const bf16* __restrict__ bin,
+                                                     const bf16* __restrict__ mod, int ldm, int shift_off,
+                                                     int scale_off, bf16* __restrict__ hb, int R, int M, int td,
+                                                     float eps) {
+  pdl_wait();
+  pdl_trigger();
+  const int r = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (r >= R) return;
+  constexpr int w = 128 * VPL;
+  ln_mod_row<VPL, INPROJ>(xh + (size_t)r * w, x + (size_t)(r < M ? r : r - M) * td, win_t, bin,
+                          mod + (size_t)r * ldm, shift_off, scale_off, hb + (size_t)r * w, td, eps, lane);
 }
 
 // Schedule constants of one kept step: mean = a_x x - a_eps eps; the log
@@ -190,19 +200,29 @@ struct StepConst {
 // One CTA per token m: final LayerNorm + modulation of rows m (cond) and
 // M + m (uncond), the output projection [eps, v] of both, guidance and the
 // sampler update of x[m]. With `eval_out` the raw outputs of both rows are
-// written there instead and x is left alone.
+// written there instead and x is left alone. With next_mod the CTA then runs
+// the next kept step's block-0 input projection, LayerNorm and modulation of
+// both rows from the updated x (ln_mod_row with that step's modulations), so
+// the next network evaluation starts at its first GEMM: xh and hb rows of
+// the token hold what ln_mod_kernel would write. xh_next is xh itself, so
+// neither is restrict: the CTA reads its two rows before the barrier that
+// precedes their rewrite.
 constexpr int FIN_THREADS = 256;
-__global__ void __launch_bounds__(FIN_THREADS, 2) final_kernel(const float* __restrict__ xh, const bf16* __restrict__ mod,
+template <int VPL>
+__global__ void __launch_bounds__(FIN_THREADS, 2) final_kernel(const float* xh, const bf16* __restrict__ mod,
                                                             int ldm, int shift_off, int scale_off,
                                                             const bf16* __restrict__ wout, const float* __restrict__ bout,
                                                             int M, int w, int td, float eps, StepConst sc,
                                                             const float* __restrict__ params, float* __restrict__ x,
                                                             const float* __restrict__ noise, float* __restrict__ x_done,
-                                                            float* __restrict__ eval_out) {
+                                                            float* __restrict__ eval_out, const bf16* __restrict__ next_mod,
+                                                            const bf16* __restrict__ win_t, const bf16* __restrict__ bin,
+                                                            float* xh_next, bf16* __restrict__ hb) {
   extern __shared__ float sm[];
   float* h = sm;                        // [2][w] modulated rows
   float* o = sm + 2 * w;                // [2][2 td] outputs
   float* red = o + 4 * td;              // [2][FIN_THREADS / 32] partial sums
+  float* xs = red + 2 * (FIN_THREADS / 32);  // [td] the updated latent
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int NWARP = FIN_THREADS / 32;
   // The output weights (no kernel writes them) of this warp's output columns
@@ -313,6 +333,15 @@ __global__ void __launch_bounds__(FIN_THREADS, 2) final_kernel(const float* __re
     }
     x[(size_t)m * td + k] = nx;
     if (x_done) x_done[(size_t)m * td + k] = nx;
+    xs[k] = nx;
+  }
+  if (next_mod) {
+    __syncthreads();
+    if (warp < 2) {
+      const int r = warp == 0 ? m : M + m;
+      ln_mod_row<VPL, true>(xh_next + (size_t)r * w, xs, win_t, bin, next_mod + (size_t)r * ldm, 0, w,
+                            hb + (size_t)r * w, td, eps, lane);
+    }
   }
 }
 
@@ -443,6 +472,29 @@ cudaError_t launch_ln_mod(const Ctx& c, lazymar_head* h, const bf16* mod, bool i
   }
 }
 
+template <int VPL>
+cudaError_t launch_final_t(const Ctx& c, lazymar_head* h, size_t smem, const bf16* mod, int fshift, int fscale, int M,
+                           const hd::StepConst& sc, const float* noise, float* x_done, float* eval_out,
+                           const bf16* next_mod) {
+  return launch_pdl(hd::final_kernel<VPL>, dim3(M), dim3(hd::FIN_THREADS), smem, c.stream, (const float*)h->xh, mod,
+                    h->nmod, fshift, fscale, (const bf16*)h->out_w, (const float*)h->out_b, M, h->w, h->td,
+                    h->cfg.ln_eps, sc, (const float*)h->params, h->x, noise, x_done, eval_out, next_mod,
+                    (const bf16*)h->in_wt, (const bf16*)h->in_b, h->xh, h->hb);
+}
+
+cudaError_t launch_final(const Ctx& c, lazymar_head* h, size_t smem, const bf16* mod, int fshift, int fscale, int M,
+                         const hd::StepConst& sc, const float* noise, float* x_done, float* eval_out,
+                         const bf16* next_mod) {
+  switch (h->w / 128) {
+#define LM_FIN(V) \
+  case V: return launch_final_t<V>(c, h, smem, mod, fshift, fscale, M, sc, noise, x_done, eval_out, next_mod);
+    LM_FIN(1) LM_FIN(2) LM_FIN(3) LM_FIN(4) LM_FIN(5) LM_FIN(6) LM_FIN(7) LM_FIN(8)
+    LM_FIN(9) LM_FIN(10) LM_FIN(11) LM_FIN(12) LM_FIN(13) LM_FIN(14) LM_FIN(15) LM_FIN(16)
+#undef LM_FIN
+    default: return cudaErrorInvalidValue;
+  }
+}
+
 // Gathers the z rows and embeds them (W_c z + b_c), once per call.
 lazymar_status prologue(lazymar_head* h, const Ctx& c, const void* z, int B, int n_img, int n_new, int M) {
   const int R = 2 * M, cd = h->cfg.cond_dim;
@@ -478,12 +530,17 @@ lazymar_status modulations(lazymar_head* h, const Ctx& c, int M, int j0, int cnt
 // One network evaluation at kept step j on rows [x; x] with its modulations
 // `mod` (R rows of nmod); ends with the final kernel (sampler update, or raw
 // outputs to eval_out).
-lazymar_status network(lazymar_head* h, const Ctx& c, int M, int j, const bf16* mod, bool done, float* eval_out) {
+// With first_done the block-0 rows were already computed by the previous
+// step's final kernel; with next_mod this step's final kernel computes them
+// for the next kept step (whose modulations are next_mod).
+lazymar_status network(lazymar_head* h, const Ctx& c, int M, int j, const bf16* mod, bool done, float* eval_out,
+                       bool first_done = false, const bf16* next_mod = nullptr) {
   const int R = 2 * M, w = h->w, depth = h->cfg.depth, td = h->td;
   for (int b = 0; b < depth; ++b) {
-    HD_TRY(hlaunch(h, b == 0 ? 2.0 * R * td * w : 0.0, "head layernorm", [&] {
-      return launch_ln_mod(c, h, mod, b == 0, R, M, 3 * w * b, 3 * w * b + w);
-    }));
+    if (b > 0 || !first_done)
+      HD_TRY(hlaunch(h, b == 0 ? 2.0 * R * td * w : 0.0, "head layernorm", [&] {
+        return launch_ln_mod(c, h, mod, b == 0, R, M, 3 * w * b, 3 * w * b + w);
+      }));
     HD_TRY(hgemm(h, c, h->hb, h->w1[b], R, w, w,
                  GemmEpi{LAZYMAR_EPI_SILU, h->b1[b], h->u, w, nullptr, nullptr, nullptr, 0}));
     GemmEpi e2{LAZYMAR_EPI_RESIDUAL, h->b2[b], h->xh, w, nullptr, nullptr, nullptr, 0};
@@ -493,13 +550,12 @@ lazymar_status network(lazymar_head* h, const Ctx& c, int M, int j, const bf16* 
   }
   const hd::StepConst sc = h->sched[j];
   const int fshift = 3 * w * depth, fscale = fshift + w;
-  const size_t smem = (size_t)(2 * w + 4 * td + 2 * (hd::FIN_THREADS / 32)) * sizeof(float);
-  return hlaunch(h, 2.0 * R * 2 * td * w, "head final", [&] {
-    return launch_pdl(hd::final_kernel, dim3(M), dim3(hd::FIN_THREADS), smem, c.stream, (const float*)h->xh, mod,
-                      h->nmod, fshift, fscale, (const bf16*)h->out_w, (const float*)h->out_b, M, w, td,
-                      h->cfg.ln_eps, sc, (const float*)h->params, h->x,
-                      (const float*)(h->noise + (size_t)(h->cfg.n_steps - 1 - j + (sc.last ? 0 : 1)) * M * td),
-                      done ? h->x_done : nullptr, eval_out);
+  const size_t smem = (size_t)(2 * w + 4 * td + 2 * (hd::FIN_THREADS / 32) + td) * sizeof(float);
+  const double flops = 2.0 * R * 2 * td * w + (next_mod ? 2.0 * R * td * w : 0.0);
+  return hlaunch(h, flops, "head final", [&] {
+    return launch_final(c, h, smem, mod, fshift, fscale, M, sc,
+                        (const float*)(h->noise + (size_t)(h->cfg.n_steps - 1 - j + (sc.last ? 0 : 1)) * M * td),
+                        done ? h->x_done : nullptr, eval_out, next_mod);
   });
 }
 
@@ -511,8 +567,11 @@ lazymar_status sample_body(lazymar_head* h, const Ctx& c, const void* z, int B, 
   for (int j0 = h->cfg.n_steps - 1; j0 >= 0; j0 -= h->chunk) {
     const int cnt = j0 + 1 < h->chunk ? j0 + 1 : h->chunk;
     HD_TRY(modulations(h, c, M, j0, cnt));
+    // inside a chunk each final kernel also computes the next step's block-0
+    // rows, whose modulations are already there
     for (int k = 0; k < cnt; ++k)
-      HD_TRY(network(h, c, M, j0 - k, h->mod + (size_t)k * 2 * M * h->nmod, j0 - k == 0, nullptr));
+      HD_TRY(network(h, c, M, j0 - k, h->mod + (size_t)k * 2 * M * h->nmod, j0 - k == 0, nullptr, k > 0,
+                     k + 1 < cnt ? h->mod + (size_t)(k + 1) * 2 * M * h->nmod : nullptr));
   }
   return LAZYMAR_OK;
 }
