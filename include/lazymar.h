@@ -29,7 +29,13 @@
  *     for the similarity of Eq. 8).
  *   - Pointers: unless stated otherwise a tensor pointer may be device memory or
  *     host memory (pinned or pageable). Host buffers are staged through
- *     library-owned device buffers with cudaMemcpyAsync on `stream`.
+ *     library-owned device buffers on `stream`. In the step calls, inputs
+ *     the device can address (device memory, page-locked host memory mapped
+ *     under unified addressing) are gathered into the staging buffers by one
+ *     copy kernel, pageable ones by cudaMemcpyAsync; the guided output is
+ *     written by the CFG kernel straight into device memory or mapped
+ *     page-locked host memory when it starts on a 16-byte boundary, and
+ *     otherwise staged and copied out.
  *   - stream: a cudaStream_t (NULL = legacy default stream). Calls enqueue work
  *     and return without waiting; buffers must stay valid until the stream work
  *     has completed. Argument errors are returned immediately and enqueue

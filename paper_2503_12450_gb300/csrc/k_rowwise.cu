@@ -476,6 +476,39 @@ __global__ void __launch_bounds__(256) cfg_kernel(int mode, const T* __restrict_
   }
 }
 
+// Copies every segment of L, block-strided over 16-byte vectors where both
+// ends are 16-byte aligned, byte by byte for the rest.
+__global__ void __launch_bounds__(256) copy_list_kernel(const CopyList L) {
+  pdl_wait();
+  pdl_trigger();
+  const size_t t = blockIdx.x * (size_t)blockDim.x + threadIdx.x, stride = (size_t)gridDim.x * blockDim.x;
+  for (int s = 0; s < L.n; ++s) {
+    const uint8_t* src = static_cast<const uint8_t*>(L.src[s]);
+    uint8_t* dst = static_cast<uint8_t*>(L.dst[s]);
+    const size_t n = L.bytes[s];
+    size_t done = 0;
+    if (((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15u) == 0) {
+      const size_t nv = n / 16;
+      for (size_t i = t; i < nv; i += stride)
+        reinterpret_cast<uint4*>(dst)[i] = reinterpret_cast<const uint4*>(src)[i];
+      done = nv * 16;
+    }
+    for (size_t i = done + t; i < n; i += stride) dst[i] = src[i];
+  }
+}
+
+cudaError_t launch_copy_list(const Ctx& c, const CopyList& L) {
+  if (L.n <= 0) return cudaSuccess;
+  if (L.n > kMaxCopySegs) return cudaErrorInvalidValue;
+  size_t total = 0;
+  for (int s = 0; s < L.n; ++s) total += L.bytes[s];
+  size_t blocks = (total / 16 + 1023) / 1024;  // about four vectors per thread
+  const size_t cap = (size_t)c.num_sms * 2;
+  if (blocks > cap) blocks = cap;
+  if (blocks == 0) blocks = 1;
+  return launch_pdl(copy_list_kernel, dim3((unsigned)blocks), dim3(256), 0, c.stream, L);
+}
+
 cudaError_t launch_cfg(const Ctx& c, int dtype, int mode, const void* zc, const void* zu, void* delta, float gamma,
                        size_t n, void* zu_out, void* g_out) {
   if (n == 0) return cudaSuccess;

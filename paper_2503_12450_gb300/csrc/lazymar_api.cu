@@ -451,15 +451,56 @@ extern "C" void lazymar_destroy(lazymar_handle* h) {
 // ---------------------------------------------------------------------------
 namespace {
 
+// The address at which the device reads `p`: p itself for device or managed
+// memory, the mapping of page-locked host memory, else nullptr (pageable
+// host memory, which only a copy can read).
+const void* device_view(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return p;
+  if (a.type == cudaMemoryTypeHost) return a.devicePointer;
+  return nullptr;
+}
+
 // Step inputs always go through the handle's staging buffers, so the device
 // work of a step reads fixed addresses and can be replayed from a CUDA graph.
-lazymar_status stage_inputs(lazymar_handle* h, const lazymar_step_in* in, cudaStream_t st) {
+// Inputs the device can address are gathered by one copy kernel (one launch
+// on the compute stream instead of a copy-engine operation per input);
+// pageable host inputs take a copy each.
+struct Stager {
+  lazymar_handle* h;
+  cudaStream_t st;
+  CopyList L{};
+  lazymar_status add(void* dst, const void* src, size_t bytes) {
+    if (bytes == 0) return LAZYMAR_OK;
+    const void* d = device_view(src);
+    if (d && L.n < kMaxCopySegs) {
+      L.src[L.n] = d;
+      L.dst[L.n] = dst;
+      L.bytes[L.n] = bytes;
+      ++L.n;
+      return LAZYMAR_OK;
+    }
+    LM_CUDA(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDefault, st));
+    return LAZYMAR_OK;
+  }
+  lazymar_status flush(const Ctx& c) {
+    if (L.n == 0) return LAZYMAR_OK;
+    return launch(h, LAZYMAR_K_OTHER, 0, 0, c.stream, "stage inputs", [&] { return launch_copy_list(c, L); });
+  }
+};
+
+lazymar_status stage_inputs(Stager& sg, const lazymar_step_in* in) {
+  lazymar_handle* h = sg.h;
   const int B = in->batch;
   const size_t nl = (size_t)B * h->cfg.n_img * h->cfg.token_dim;
   const size_t nm = (size_t)B * h->cfg.n_img;
-  LM_CUDA(cudaMemcpyAsync(h->st_lat, in->latents, nl * 4, cudaMemcpyDefault, st));
-  LM_CUDA(cudaMemcpyAsync(h->st_mask, in->mask, nm, cudaMemcpyDefault, st));
-  LM_CUDA(cudaMemcpyAsync(h->st_labels, in->labels, (size_t)B * 4, cudaMemcpyDefault, st));
+  LM_TRY(sg.add(h->st_lat, in->latents, nl * 4));
+  LM_TRY(sg.add(h->st_mask, in->mask, nm));
+  LM_TRY(sg.add(h->st_labels, in->labels, (size_t)B * 4));
   return LAZYMAR_OK;
 }
 
@@ -584,9 +625,30 @@ lazymar_status cfg(lazymar_handle* h, const Ctx& c, int mode, int B, float gamma
   });
 }
 
-// Resolves an output pointer: device pointers are written directly, host
-// pointers through the staging buffer `st` and a copy at the end.
-void* out_target(void* user, void* st) { return user == nullptr ? nullptr : (is_device_ptr(user) ? user : st); }
+// Resolves an output pointer: device pointers on a 16-byte boundary (the
+// kernels store 16-byte vectors) are written directly, any other pointer
+// through the staging buffer `st` and a copy at the end.
+void* out_target(void* user, void* st) {
+  return user == nullptr ? nullptr : (is_device_ptr(user) && aligned16(user) ? user : st);
+}
+
+// Target of the guided output, which the CFG kernel writes: the caller's
+// buffer when it is device memory, or page-locked host memory mapped into the
+// device's address space (cudaHostAlloc / cudaHostRegister under unified
+// addressing), which the kernel then writes directly (no staging and no
+// separate device-to-host copy); otherwise the staging buffer, copied out
+// afterwards.
+void* guided_target(void* user, void* st) {
+  if (user == nullptr) return nullptr;
+  if (is_device_ptr(user)) return aligned16(user) ? user : st;
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, user) != cudaSuccess) {
+    cudaGetLastError();
+    return st;
+  }
+  if (a.type == cudaMemoryTypeHost && a.devicePointer && aligned16(a.devicePointer)) return a.devicePointer;
+  return st;
+}
 
 // Device work of a full step up to the output cache (everything but the CFG
 // combine, which takes gamma and stays outside any graph).
@@ -754,14 +816,16 @@ extern "C" lazymar_status lazymar_full_step(lazymar_handle* h, const lazymar_ste
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const Ctx c{st, h->err, h->num_sms};
   const int B = in->batch;
-  LM_TRY(stage_inputs(h, in, st));
+  Stager sg{h, st};
+  LM_TRY(stage_inputs(sg, in));
+  LM_TRY(sg.flush(c));
   LM_TRY(run_body(h, st, lazymar_handle::GraphKey{0, B, 0, 0, 0, 0}, [&](const Ctx& cc) { return full_body(h, cc, B); }));
-  void* g_dst = out_target(guided_out, h->st_g);
+  void* g_dst = guided_target(guided_out, h->st_g);
   LM_TRY(cfg(h, c, LAZYMAR_CFG_REFRESH, B, gamma, nullptr, g_dst));
   const size_t zbytes = (size_t)2 * B * h->cfg.n_img * h->D * h->es;
   if (z_out) LM_CUDA(cudaMemcpyAsync(z_out, h->zc, zbytes, cudaMemcpyDefault, st));
-  if (guided_out && g_dst != guided_out)
-    LM_CUDA(cudaMemcpyAsync(guided_out, g_dst, zbytes / 2, cudaMemcpyDeviceToHost, st));
+  if (guided_out && g_dst == h->st_g)
+    LM_CUDA(cudaMemcpyAsync(guided_out, g_dst, zbytes / 2, cudaMemcpyDefault, st));
   h->primed = true;
   h->last_batch = B;
   return LAZYMAR_OK;
@@ -779,9 +843,10 @@ extern "C" lazymar_status lazymar_cached_step(lazymar_handle* h, const lazymar_s
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const Ctx c{st, h->err, h->num_sms};
   const int B = in->batch, rows = use_cond_cache ? B : 2 * B, N = n_compute, D = h->D;
-  LM_TRY(stage_inputs(h, in, st));
+  Stager sg{h, st};
+  LM_TRY(stage_inputs(sg, in));
   const bool has_idx = idx_in != nullptr && N > 0;
-  if (has_idx) LM_CUDA(cudaMemcpyAsync(h->st_idx_in, idx_in, (size_t)rows * N * 4, cudaMemcpyDefault, st));
+  if (has_idx) LM_TRY(sg.add(h->st_idx_in, idx_in, (size_t)rows * N * 4));
   // selection inputs (Table 3 rules): priority classes and random keys
   const bool sel_rule = !has_idx && N > 0;
   const bool has_prio = sel_rule && in->select_priority != nullptr;
@@ -789,15 +854,16 @@ extern "C" lazymar_status lazymar_cached_step(lazymar_handle* h, const lazymar_s
   if (has_keys && !in->select_keys)
     return fail(LAZYMAR_ERR_INVALID_ARG, "LAZYMAR_SELECT_RANDOM needs select_keys on cached steps");
   const size_t rowsT = (size_t)rows * h->T;
-  if (has_prio) LM_CUDA(cudaMemcpyAsync(h->st_prio, in->select_priority, rowsT, cudaMemcpyDefault, st));
-  if (has_keys) LM_CUDA(cudaMemcpyAsync(h->st_keys, in->select_keys, rowsT * 4, cudaMemcpyDefault, st));
+  if (has_prio) LM_TRY(sg.add(h->st_prio, in->select_priority, rowsT));
+  if (has_keys) LM_TRY(sg.add(h->st_keys, in->select_keys, rowsT * 4));
+  LM_TRY(sg.flush(c));
   const int sel = (has_prio ? 1 : 0) | (has_keys ? 2 : 0);
   LM_TRY(run_body(h, st, lazymar_handle::GraphKey{1, B, N, use_cond_cache ? 1 : 0, has_idx ? 1 : 0, sel},
                   [&](const Ctx& cc) { return cached_body(h, cc, rows, N, has_idx, sel); }));
 
   const size_t n_el = (size_t)B * h->cfg.n_img * D;
   void* z_dst = out_target(z_out, h->st_z);
-  void* g_dst = out_target(guided_out, h->st_g);
+  void* g_dst = guided_target(guided_out, h->st_g);
   uint8_t* z8 = static_cast<uint8_t*>(z_dst);
   if (use_cond_cache) {
     LM_TRY(cfg(h, c, LAZYMAR_CFG_REUSE, B, gamma, z8 ? z8 + n_el * h->es : nullptr, g_dst));
@@ -806,9 +872,9 @@ extern "C" lazymar_status lazymar_cached_step(lazymar_handle* h, const lazymar_s
     LM_TRY(cfg(h, c, LAZYMAR_CFG_REFRESH, B, gamma, nullptr, g_dst));
     if (z8) LM_CUDA(cudaMemcpyAsync(z8, h->zc, 2 * n_el * h->es, cudaMemcpyDeviceToDevice, st));
   }
-  if (z_out && z_dst != z_out) LM_CUDA(cudaMemcpyAsync(z_out, z_dst, 2 * n_el * h->es, cudaMemcpyDeviceToHost, st));
-  if (guided_out && g_dst != guided_out)
-    LM_CUDA(cudaMemcpyAsync(guided_out, g_dst, n_el * h->es, cudaMemcpyDeviceToHost, st));
+  if (z_out && z_dst != z_out) LM_CUDA(cudaMemcpyAsync(z_out, z_dst, 2 * n_el * h->es, cudaMemcpyDefault, st));
+  if (guided_out && g_dst == h->st_g)
+    LM_CUDA(cudaMemcpyAsync(guided_out, g_dst, n_el * h->es, cudaMemcpyDefault, st));
   if (idx_out && N > 0) LM_CUDA(cudaMemcpyAsync(idx_out, h->idx, (size_t)rows * N * 4, cudaMemcpyDefault, st));
   return LAZYMAR_OK;
 }

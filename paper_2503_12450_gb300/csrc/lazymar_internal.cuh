@@ -530,6 +530,18 @@ cudaError_t launch_idx_check(const Ctx& c, const int* idx_in, int rows, int T, i
 cudaError_t launch_cfg(const Ctx& c, int dtype, int mode, const void* zc, const void* zu, void* delta,
                        float gamma, size_t n, void* zu_out, void* g_out);
 
+// Up to kMaxCopySegs byte ranges copied by one kernel (the step inputs into
+// the handle's staging buffers). Each source is device memory or page-locked
+// host memory the device can address.
+constexpr int kMaxCopySegs = 6;
+struct CopyList {
+  const void* src[kMaxCopySegs];
+  void* dst[kMaxCopySegs];
+  unsigned long long bytes[kMaxCopySegs];
+  int n;
+};
+cudaError_t launch_copy_list(const Ctx& c, const CopyList& L);
+
 // NVTX range for the lifetime of the object (header-only NVTX v3: a no-op
 // unless a profiler has attached its tool library).
 struct NvtxRange {

@@ -248,6 +248,28 @@ def test_host_buffers_match_device_buffers(tiny):
     lm.lazymar_cached_step(r.h, lat1, m1, r.labels, 1, N, False, GAMMA, None, ih, zh, gh)
     lm.lazymar_sync(r.h)
     assert np.array_equal(zh, zd) and np.array_equal(gh, gd) and np.array_equal(ih, Id)
+    # page-locked host outputs (the guided output is written by the kernel
+    # through the mapping) and device outputs off a 16-byte boundary (staged)
+    torch = torch_cuda()
+    zp = torch.zeros(tuple(zh.shape), dtype=torch.float32).pin_memory()
+    gp = torch.zeros(tuple(gh.shape), dtype=torch.float32).pin_memory()
+    zo = torch.zeros(zh.size + 1, device="cuda")[1:].view(zh.shape)
+    go = torch.zeros(gh.size + 1, device="cuda")[1:].view(gh.shape)
+    assert zo.data_ptr() % 16 and go.data_ptr() % 16
+    for z_out, g_out in ((zp, gp), (zo, go)):
+        lm.lazymar_full_step(r.h, lat0, m0, r.labels, 1, GAMMA, z_out, g_out)
+        lm.lazymar_cached_step(r.h, lat1, m1, r.labels, 1, N, False, GAMMA, None, None, z_out, g_out)
+        lm.lazymar_sync(r.h)
+        assert np.array_equal(z_out.cpu().numpy(), zd) and np.array_equal(g_out.cpu().numpy(), gd)
+    # a condition-reuse step writes the unconditional half of z through the
+    # same targets
+    zr, gr, _ = r.cached((lat1, m1), N, True)
+    lm.lazymar_full_step(r.h, lat0, m0, r.labels, 1, GAMMA)
+    lm.lazymar_cached_step(r.h, lat1, m1, r.labels, 1, N, False, GAMMA)
+    for z_out, g_out in ((zp, gp), (zo, go)):
+        lm.lazymar_cached_step(r.h, lat1, m1, r.labels, 1, N, True, GAMMA, None, None, z_out, g_out)
+        lm.lazymar_sync(r.h)
+        assert np.array_equal(z_out.cpu().numpy(), zr) and np.array_equal(g_out.cpu().numpy(), gr)
 
 
 def test_step_state_and_device_errors():
