@@ -403,6 +403,7 @@ def test_linear_e4m3(M, N, K, epi):
     (2, 320, 320, 16, 80, "bf16", 1.0),   # MAR-H full layer (three query tiles)
     (2, 65, 130, 2, 80, "bf16", 1.0),     # ragged queries and keys
     (1, 129, 200, 3, 80, "bf16", 1.0),    # one query past a tile, a ragged key chunk
+    (3, 256, 300, 5, 64, "bf16", 1.0),    # whole query tiles only (no shorter last tile)
     (1, 1, 1, 1, 80, "bf16", 1.0),
     (1, 1, 1, 1, 64, "bf16", 1.0),
     # scores of std ~6 (log2 units): the running maximum is raised mid-row
