@@ -155,8 +155,7 @@ struct lazymar_handle {
   // events of a short kernel).
   std::map<GraphKey, GraphEntry> pgraphs;
   bool use_graphs = true;
-  cudaStream_t gstream = nullptr;  // capture / replay stream
-  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  cudaStream_t gstream = nullptr;  // capture stream (graphs replay on the caller's stream)
 };
 
 namespace {
@@ -388,10 +387,8 @@ extern "C" lazymar_status lazymar_create(const lazymar_config* cfg, const lazyma
 
   e = cudaMemset(h->arena, 0, h->arena_bytes);
   if (e != cudaSuccess) return destroy(cuda_fail(e, "cudaMemset"));
-  if ((e = cudaStreamCreateWithFlags(&h->gstream, cudaStreamNonBlocking)) != cudaSuccess ||
-      (e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming)) != cudaSuccess ||
-      (e = cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming)) != cudaSuccess)
-    return destroy(cuda_fail(e, "stream/event creation"));
+  if ((e = cudaStreamCreateWithFlags(&h->gstream, cudaStreamNonBlocking)) != cudaSuccess)
+    return destroy(cuda_fail(e, "stream creation"));
   lazymar_status st;
   const int dt = cfg->dtype;
   if ((st = upload(h->pos, w->pos_emb, T * D, dt)) || (st = upload(h->cls, w->class_emb, (size_t)cfg->n_classes * D, dt)) ||
@@ -435,8 +432,6 @@ extern "C" void lazymar_destroy(lazymar_handle* h) {
       cudaEventDestroy(e.b);
     }
   }
-  if (h->ev_fork) cudaEventDestroy(h->ev_fork);
-  if (h->ev_join) cudaEventDestroy(h->ev_join);
   if (h->gstream) cudaStreamDestroy(h->gstream);
   for (auto& e : h->evs) {
     cudaEventDestroy(e.a);
@@ -768,9 +763,9 @@ lazymar_status run_body(lazymar_handle* h, cudaStream_t st, const lazymar_handle
   lazymar_handle::GraphEntry& ge = h->profiling ? h->pgraphs[key] : h->graphs[key];
   if (!h->profiling && !ge.exec && ge.eager_runs++ == 0) return body(Ctx{st, h->err, h->num_sms});
   LM_TRY(drain_profiled(h, ge));
+  // captured on the handle's own stream (the caller's may be the legacy
+  // stream, which cannot be captured), replayed on the caller's stream
   cudaStream_t gs = h->gstream;
-  LM_CUDA(cudaEventRecord(h->ev_fork, st));
-  LM_CUDA(cudaStreamWaitEvent(gs, h->ev_fork, 0));
   if (!ge.exec) {
     const lazymar_stats before = h->stats;
     const size_t ev_base = h->ev_used;
@@ -798,9 +793,7 @@ lazymar_status run_body(lazymar_handle* h, cudaStream_t st, const lazymar_handle
     add_stats(ge.delta, before, -1.0);
     h->stats = before;
   }
-  LM_CUDA(cudaGraphLaunch(ge.exec, gs));
-  LM_CUDA(cudaEventRecord(h->ev_join, gs));
-  LM_CUDA(cudaStreamWaitEvent(st, h->ev_join, 0));
+  LM_CUDA(cudaGraphLaunch(ge.exec, st));
   add_stats(h->stats, ge.delta, 1.0);
   ge.pending = h->profiling;
   return LAZYMAR_OK;
