@@ -333,8 +333,9 @@ lazymar_status lazymar_read_reference(lazymar_handle *h, int rows, void *dst, vo
  * fixed addresses. That work (embedding through the final LayerNorm) runs
  * eagerly the first time a (step kind, B, N, cond reuse, idx_in given)
  * combination is seen, is captured into a CUDA graph the second time (on a
- * stream of the handle's) and replayed on `stream` from then on; the CFG combine and the output copies are launched
- * after it, so gamma may change from call to call. enable = 0 runs every step
+ * stream of the handle's) and replayed on `stream` from then on; the CFG
+ * combine and the output copies are launched after it, so gamma may change
+ * from call to call. enable = 0 runs every step
  * eagerly. While profiling is on, each combination is captured on its first
  * use together with an event record around every launch, into a graph of its
  * own, and replayed; the per-kernel times are then device times, free of the
