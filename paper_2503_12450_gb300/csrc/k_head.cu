@@ -5,14 +5,16 @@
 //
 // One sampling call runs, for the R = 2M rows (M tokens x {cond, uncond}):
 //   gather z rows -> W_c z + b_c (tcgen05 GEMM)                      once
+//   per chunk of kept steps (they depend on the embeddings only):
+//     SiLU(t_emb[j] + c_emb) for every step j of the chunk  (row-wise)
+//     all blocks' and the final modulations of those steps  (one tcgen05 GEMM)
 //   per kept step j = n_steps-1 .. 0:
-//     SiLU(t_emb[j] + c_emb)                                (row-wise)
-//     all blocks' and the final modulations in one GEMM     (tcgen05, bias)
-//     block 0: input projection + LN + modulation           (row-wise)
+//     block 0: input projection + LN + modulation           (row-wise; inside
+//              a chunk done by the previous step's final kernel)
 //     per block: fc1 + SiLU (GEMM), fc2 gated into the fp32 residual (GEMM),
 //                next LN + modulation                        (row-wise)
-//     final LN + modulation, output projection, guidance and the sampler
-//     update of x                                            (one CTA per token)
+//     final LN + modulation, output projection, guidance, the sampler
+//     update of x, and the next step's block-0 rows          (one CTA per token)
 // The loop runs eagerly on the first call with a given (z buffer, B, n_img,
 // n_new), is captured into a CUDA graph on the second and replayed after that.
 // The guidance scale and temperature are read from device memory, so they may
